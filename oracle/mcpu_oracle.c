@@ -1,0 +1,324 @@
+/*
+ * CPU oracle for the paged-attention hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY. Nothing in the product path links, loads or calls
+ * this file: only the tests, the smoke check and the bench's CPU-baseline leg
+ * use it. It shares no code, header or constant with the CUDA library.
+ *
+ * What it computes. The paper (§3.2) names generation -- autoregressive
+ * decoding of hundreds of concurrent multi-turn trajectories, with tool
+ * observations appended between turns -- as the GPU-bound stage of a rollout
+ * step; the G = 8 samples of a GRPO task (§4, App. B Tab. "hparams") share
+ * their prompt. The paper prints no attention formula, so the operation is the
+ * textbook one, written out exactly as defined and in the most direct order:
+ *
+ *   1. kv append:  for row r with L_r new tokens and post-append length S_r,
+ *      new token i (0 <= i < L_r) lands at position pos = S_r - L_r + i, i.e.
+ *      physical page block_table[r][pos / page] at slot pos % page, for K and
+ *      for V, bit for bit.
+ *   2. attention:  query i of row r sits at position p = S_r - L_r + i. Key j
+ *      of the row is gathered from page block_table[r][j / page], slot
+ *      j % page. Key j is visible iff j <= p (causal) and, when the sliding
+ *      window W > 0, p - j < W. With q head h reading kv head h / (H_q/H_kv):
+ *         s_j  = scale * sum_d q[d] * K[j][d]
+ *         m    = max_j s_j,   l = sum_j exp(s_j - m)
+ *         out  = sum_j exp(s_j - m) / l * V[j]          (rounded to bf16)
+ *         lse  = m + ln(l)    (natural log of sum_j exp(s_j))
+ *      A query with no visible key has out = 0 and lse = -inf.
+ *
+ * Precision: bf16 inputs are widened exactly; every sum and product is taken
+ * in double; out is rounded once, double -> bf16, to nearest-even.
+ *
+ * Layouts (all row-major, bf16 passed as its uint16 bit pattern):
+ *   q        [T_q, H_q, D]            k_new, v_new [T_q, H_kv, D]
+ *   k_cache  [num_pages, H_kv, page, D]   (same for v_cache)
+ *   block_table [num_seqs, max_pages_per_seq] int32
+ *   seq_lens [num_seqs] int32,  query_start_loc [num_seqs + 1] int32
+ *   out [T_q, H_q, D] bf16 bits,  lse [T_q, H_q] float
+ *
+ * Return value: 0 on success, otherwise a positive code naming the first
+ * problem found (see ORACLE_ERR_*); nothing is written past a failed check.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORACLE_OK 0
+#define ORACLE_ERR_SHAPE 1     /* bad dims, or query_start_loc not monotone */
+#define ORACLE_ERR_LENGTH 2    /* L_r > S_r, S_r < 0, or S_r beyond the table */
+#define ORACLE_ERR_PAGE 3      /* a page that must be read or written is out of range */
+#define ORACLE_ERR_NOMEM 4
+
+static double bf16_to_double(uint16_t b) {
+  uint32_t u = (uint32_t)b << 16;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return (double)f;
+}
+
+/* Round a double to the nearest bf16 (8 significant bits, exponent range of
+ * float), ties to even. Written from the definition: pick the quantum of the
+ * binade (or the subnormal quantum 2^-133), round the scaled value with rint
+ * (nearest-even in the default rounding mode), scale back. */
+uint16_t oracle_double_to_bf16(double x) {
+  if (isnan(x)) return 0x7FC0;
+  double ax = fabs(x);
+  double r;
+  if (ax == 0.0) {
+    r = 0.0;
+  } else {
+    int e;
+    frexp(ax, &e);          /* ax = m * 2^e, 0.5 <= m < 1 */
+    int qexp = e - 8;       /* 8 significant bits -> quantum 2^(e-8) */
+    if (qexp < -133) qexp = -133;
+    r = ldexp(rint(ldexp(ax, -qexp)), qexp);
+  }
+  float f = (float)r; /* exact (or +inf on overflow) */
+  if (x < 0) f = -f;
+  uint32_t u;
+  memcpy(&u, &f, sizeof u);
+  return (uint16_t)(u >> 16);
+}
+
+static int check_common(const int32_t* seq_lens, const int32_t* qsl, int32_t num_seqs,
+                        int32_t max_pages_per_seq, int32_t num_q_heads, int32_t num_kv_heads,
+                        int32_t head_dim, int32_t page_size) {
+  if (num_seqs < 0 || max_pages_per_seq < 0 || num_kv_heads <= 0 || num_q_heads <= 0 ||
+      head_dim <= 0 || page_size <= 0 || num_q_heads % num_kv_heads != 0)
+    return ORACLE_ERR_SHAPE;
+  if (num_seqs > 0 && qsl[0] != 0) return ORACLE_ERR_SHAPE;
+  for (int32_t r = 0; r < num_seqs; ++r) {
+    int64_t L = (int64_t)qsl[r + 1] - qsl[r];
+    int64_t S = seq_lens[r];
+    if (L < 0) return ORACLE_ERR_SHAPE;
+    if (S < 0 || L > S) return ORACLE_ERR_LENGTH;
+    if (S > (int64_t)max_pages_per_seq * page_size) return ORACLE_ERR_LENGTH;
+  }
+  return ORACLE_OK;
+}
+
+/* Step 1: scatter the new K/V rows of every query token into the pools. */
+int oracle_kv_append(const uint16_t* k_new, const uint16_t* v_new, uint16_t* k_cache,
+                     uint16_t* v_cache, const int32_t* block_table, const int32_t* seq_lens,
+                     const int32_t* query_start_loc, int32_t num_seqs,
+                     int32_t max_pages_per_seq, int64_t num_pages, int32_t num_kv_heads,
+                     int32_t head_dim, int32_t page_size) {
+  int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_kv_heads,
+                        num_kv_heads, head_dim, page_size);
+  if (rc) return rc;
+  /* Check every destination page before writing anything. */
+  for (int32_t r = 0; r < num_seqs; ++r) {
+    int64_t L = query_start_loc[r + 1] - query_start_loc[r];
+    int64_t S = seq_lens[r];
+    for (int64_t i = 0; i < L; ++i) {
+      int64_t pos = S - L + i;
+      int64_t page = block_table[(int64_t)r * max_pages_per_seq + pos / page_size];
+      if (page < 0 || page >= num_pages) return ORACLE_ERR_PAGE;
+    }
+  }
+  for (int32_t r = 0; r < num_seqs; ++r) {
+    int64_t L = query_start_loc[r + 1] - query_start_loc[r];
+    int64_t S = seq_lens[r];
+    for (int64_t i = 0; i < L; ++i) {
+      int64_t tok = query_start_loc[r] + i;
+      int64_t pos = S - L + i;
+      int64_t page = block_table[(int64_t)r * max_pages_per_seq + pos / page_size];
+      int64_t slot = pos % page_size;
+      for (int32_t h = 0; h < num_kv_heads; ++h) {
+        const uint16_t* ks = k_new + (tok * num_kv_heads + h) * head_dim;
+        const uint16_t* vs = v_new + (tok * num_kv_heads + h) * head_dim;
+        uint16_t* kd = k_cache + ((page * num_kv_heads + h) * page_size + slot) * head_dim;
+        uint16_t* vd = v_cache + ((page * num_kv_heads + h) * page_size + slot) * head_dim;
+        for (int32_t d = 0; d < head_dim; ++d) {
+          kd[d] = ks[d];
+          vd[d] = vs[d];
+        }
+      }
+    }
+  }
+  return ORACLE_OK;
+}
+
+/* Visible key range [lo, p] of a query at position p (step 2's mask). */
+static int64_t first_visible(int64_t p, int32_t window) {
+  if (window <= 0) return 0;
+  int64_t lo = p - window + 1;
+  return lo < 0 ? 0 : lo;
+}
+
+/* Step 2 for one query vector: gathers its visible keys straight from the
+ * pages and writes out[0..D) (bf16 bits) and *lse. */
+static int attend_one(const uint16_t* qv, const uint16_t* k_cache, const uint16_t* v_cache,
+                      const int32_t* bt_row, int64_t p, int32_t kvh, int32_t window,
+                      double scale, int64_t num_pages, int32_t num_kv_heads, int32_t head_dim,
+                      int32_t page_size, double* s, double* acc, uint16_t* out, float* lse) {
+  int64_t lo = first_visible(p, window);
+  int64_t n = p - lo + 1;
+  if (n <= 0) {
+    for (int32_t d = 0; d < head_dim; ++d) out[d] = 0;
+    *lse = -INFINITY;
+    return ORACLE_OK;
+  }
+  /* scores */
+  double m = -INFINITY;
+  for (int64_t j = lo; j <= p; ++j) {
+    int64_t page = bt_row[j / page_size];
+    if (page < 0 || page >= num_pages) return ORACLE_ERR_PAGE;
+    const uint16_t* kj = k_cache + ((page * num_kv_heads + kvh) * page_size + j % page_size) * head_dim;
+    double dot = 0.0;
+    for (int32_t d = 0; d < head_dim; ++d) dot += bf16_to_double(qv[d]) * bf16_to_double(kj[d]);
+    s[j - lo] = scale * dot;
+    if (s[j - lo] > m) m = s[j - lo];
+  }
+  /* normaliser */
+  double l = 0.0;
+  for (int64_t j = 0; j < n; ++j) l += exp(s[j] - m);
+  /* weighted sum of values */
+  for (int32_t d = 0; d < head_dim; ++d) acc[d] = 0.0;
+  for (int64_t j = lo; j <= p; ++j) {
+    int64_t page = bt_row[j / page_size];
+    const uint16_t* vj = v_cache + ((page * num_kv_heads + kvh) * page_size + j % page_size) * head_dim;
+    double w = exp(s[j - lo] - m) / l;
+    for (int32_t d = 0; d < head_dim; ++d) acc[d] += w * bf16_to_double(vj[d]);
+  }
+  for (int32_t d = 0; d < head_dim; ++d) out[d] = oracle_double_to_bf16(acc[d]);
+  *lse = (float)(m + log(l));
+  return ORACLE_OK;
+}
+
+static int row_of_token(const int32_t* qsl, int32_t num_seqs, int64_t t) {
+  for (int32_t r = 0; r < num_seqs; ++r)
+    if (t >= qsl[r] && t < qsl[r + 1]) return r;
+  return -1;
+}
+
+/* Full attention: every query token of every row, every q head.
+ * num_threads <= 0 uses the OpenMP default. */
+int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
+                           const int32_t* block_table, const int32_t* seq_lens,
+                           const int32_t* query_start_loc, int32_t num_seqs,
+                           int32_t max_pages_per_seq, int64_t num_pages, int32_t num_q_heads,
+                           int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
+                           int32_t sliding_window, double softmax_scale, uint16_t* out,
+                           float* lse, int32_t num_threads) {
+  int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_q_heads,
+                        num_kv_heads, head_dim, page_size);
+  if (rc) return rc;
+  int64_t max_s = 1;
+  for (int32_t r = 0; r < num_seqs; ++r)
+    if (seq_lens[r] > max_s) max_s = seq_lens[r];
+  const int32_t group = num_q_heads / num_kv_heads;
+  const int64_t total_q = num_seqs > 0 ? query_start_loc[num_seqs] : 0;
+  int err = ORACLE_OK;
+#ifdef _OPENMP
+  if (num_threads > 0) omp_set_num_threads(num_threads);
+#else
+  (void)num_threads;
+#endif
+#pragma omp parallel
+  {
+    double* s = (double*)malloc(sizeof(double) * (size_t)max_s);
+    double* acc = (double*)malloc(sizeof(double) * (size_t)head_dim);
+    if (!s || !acc) {
+#pragma omp atomic write
+      err = ORACLE_ERR_NOMEM;
+    }
+#pragma omp for schedule(dynamic, 1) collapse(2)
+    for (int64_t t = 0; t < total_q; ++t) {
+      for (int32_t h = 0; h < num_q_heads; ++h) {
+        if (!s || !acc) continue;
+        int32_t r = row_of_token(query_start_loc, num_seqs, t);
+        int64_t S = seq_lens[r];
+        int64_t L = query_start_loc[r + 1] - query_start_loc[r];
+        int64_t p = S - L + (t - query_start_loc[r]);
+        int e = attend_one(q + (t * num_q_heads + h) * head_dim, k_cache, v_cache,
+                           block_table + (int64_t)r * max_pages_per_seq, p, h / group,
+                           sliding_window, softmax_scale, num_pages, num_kv_heads, head_dim,
+                           page_size, s, acc, out + (t * num_q_heads + h) * head_dim,
+                           lse + t * num_q_heads + h);
+        if (e) {
+#pragma omp atomic write
+          err = e;
+        }
+      }
+    }
+    free(s);
+    free(acc);
+  }
+  return err;
+}
+
+/* The same definition evaluated only at listed (token, q head) pairs, for
+ * spot checks of workloads too large to run in full. out_samples is
+ * [n_samples, D] bf16 bits, lse_samples [n_samples]. */
+int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
+                                   const uint16_t* v_cache, const int32_t* block_table,
+                                   const int32_t* seq_lens, const int32_t* query_start_loc,
+                                   int32_t num_seqs, int32_t max_pages_per_seq, int64_t num_pages,
+                                   int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                   int32_t page_size, int32_t sliding_window,
+                                   double softmax_scale, const int64_t* sample_token,
+                                   const int32_t* sample_head, int64_t n_samples,
+                                   uint16_t* out_samples, float* lse_samples,
+                                   int32_t num_threads) {
+  int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_q_heads,
+                        num_kv_heads, head_dim, page_size);
+  if (rc) return rc;
+  const int64_t total_q = num_seqs > 0 ? query_start_loc[num_seqs] : 0;
+  for (int64_t i = 0; i < n_samples; ++i)
+    if (sample_token[i] < 0 || sample_token[i] >= total_q || sample_head[i] < 0 ||
+        sample_head[i] >= num_q_heads)
+      return ORACLE_ERR_SHAPE;
+  int64_t max_s = 1;
+  for (int32_t r = 0; r < num_seqs; ++r)
+    if (seq_lens[r] > max_s) max_s = seq_lens[r];
+  const int32_t group = num_q_heads / num_kv_heads;
+  int err = ORACLE_OK;
+#ifdef _OPENMP
+  if (num_threads > 0) omp_set_num_threads(num_threads);
+#else
+  (void)num_threads;
+#endif
+#pragma omp parallel
+  {
+    double* s = (double*)malloc(sizeof(double) * (size_t)max_s);
+    double* acc = (double*)malloc(sizeof(double) * (size_t)head_dim);
+    if (!s || !acc) {
+#pragma omp atomic write
+      err = ORACLE_ERR_NOMEM;
+    }
+#pragma omp for schedule(dynamic, 1)
+    for (int64_t i = 0; i < n_samples; ++i) {
+      if (!s || !acc) continue;
+      int64_t t = sample_token[i];
+      int32_t h = sample_head[i];
+      int32_t r = row_of_token(query_start_loc, num_seqs, t);
+      int64_t S = seq_lens[r];
+      int64_t L = query_start_loc[r + 1] - query_start_loc[r];
+      int64_t p = S - L + (t - query_start_loc[r]);
+      int e = attend_one(q + (t * num_q_heads + h) * head_dim, k_cache, v_cache,
+                         block_table + (int64_t)r * max_pages_per_seq, p, h / group,
+                         sliding_window, softmax_scale, num_pages, num_kv_heads, head_dim,
+                         page_size, s, acc, out_samples + i * head_dim, lse_samples + i);
+      if (e) {
+#pragma omp atomic write
+        err = e;
+      }
+    }
+    free(s);
+    free(acc);
+  }
+  return err;
+}
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
