@@ -1,0 +1,562 @@
+#!/usr/bin/env python
+"""Benchmark of the paged-attention hot path on one GB300 (or N replicas).
+
+One step = one pass of the whole path over one synthetic batch: KV append of
+every query token's new K/V, then paged attention (device planner, cascade
+pass over shared GRPO prompts, split-KV decode, causal append-chunk kernel,
+log-sum-exp merge) -- for every layer of the workload.
+
+Default workload: the mixed multi-turn batch (256 trajectories with prior
+context uniform in [4096, 32768]; 224 decode one token, 32 append a tool
+observation of log-uniform length in [64, 2048]; 64 q / 8 kv heads, head dim
+64, page 16, bf16). Inputs are resident in HBM when timing starts and are far
+larger than L2 (the KV pool alone is ~10 GB), so no L2 flush is needed.
+
+Metric: KV-read GB/s = algorithmic KV bytes per step / step time, where the
+algorithmic KV bytes count every (row, key position) that some query of the
+row may see once (shared prompt pages once per group): 2 * H_kv * D * 2 bytes
+per token. Attended tokens/s (sum over queries of visible keys) is reported
+beside it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload mixed|decode|long|rollout|tiny]
+
+Prints one JSON line (rank 0). Under torchrun each rank runs an independent
+replica on its own GPU (the path has no exchange step); value is the total
+over ranks divided by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+KV_TOKEN_BYTES = lambda b: 2 * b.num_kv_heads * b.head_dim * 2  # noqa: E731
+WORKLOAD_DESC = {
+    "tiny": "tiny decode: 4 rows, S={17,64,129,300}, 8q/2kv heads, D=64, page 16, bf16",
+    "decode": "decode batch: 64 rows, S~U[2048,16384], 64q/8kv, D=64, page 16, bf16",
+    "mixed": "mixed multi-turn batch: 256 rows, prior~U[4096,32768], 224 decode + 32 append rows "
+             "(chunk logU[64,2048]), 64q/8kv, D=64, page 16, bf16",
+    "long": "long-horizon decode: 512 rows, S lognormal(median 12288, sigma 1) in [512,65536], "
+            "1/3 in [49152,65536], 64q/8kv, D=64, page 16, bf16",
+    "rollout": "rollout step: 24 layers alternating SWA-128/full, 48 GRPO groups x 8 rows sharing prompt "
+               "pages (prompt U[1024,8192], continuation U[0,24576]), 15% append rows (logU[64,1024]), "
+               "64q/8kv, D=64, page 16, bf16",
+}
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# --------------------------------------------------------------- accounting
+
+
+def layer_stats(batch: W.Batch, layer: int):
+    """Algorithmic work of one layer: KV bytes (distinct visible tokens, shared
+    prompt pages once per group), attended (query, key) pairs, split by
+    decode / append rows."""
+    lay = batch.layers[layer]
+    Wn = lay.sliding_window
+    S = batch.seq_lens.astype(np.int64)
+    L = batch.q_lens.astype(np.int64)
+    first = np.where(Wn > 0, np.maximum(0, S - L - Wn + 1), 0) if Wn > 0 else np.zeros_like(S)
+    distinct = np.where(L > 0, S - first, 0)
+    # attended pairs per row: sum_i min(p_i + 1, W)
+    pairs = np.zeros_like(S)
+    for r in range(len(S)):
+        if L[r] == 0:
+            continue
+        p = np.arange(S[r] - L[r], S[r])
+        vis = p + 1 if Wn <= 0 else np.minimum(p + 1, Wn)
+        pairs[r] = int(vis.sum())
+    shared_tokens = 0
+    if Wn <= 0 and batch.group_of_row is not None:
+        bt = batch.pools[lay.pool].block_table
+        for g in np.unique(batch.group_of_row):
+            rows = np.nonzero(batch.group_of_row == g)[0]
+            rows = rows[L[rows] > 0]
+            if len(rows) < 2:
+                continue
+            n = 0
+            ref = bt[rows[0]]
+            lim = int(min(S[rows]) // batch.page_size)
+            while n < lim and all(bt[r, n] == ref[n] for r in rows):
+                n += 1
+            shared_tokens += (len(rows) - 1) * n * batch.page_size
+    tb = KV_TOKEN_BYTES(batch)
+    dec = L == 1
+    app = L > 1
+    return dict(
+        kv_bytes=int((distinct.sum() - shared_tokens) * tb),
+        kv_bytes_decode=int(distinct[dec].sum() * tb),
+        kv_bytes_append=int(distinct[app].sum() * tb),
+        shared_tokens_saved=int(shared_tokens),
+        pairs=int(pairs.sum()),
+        pairs_decode=int(pairs[dec].sum()),
+        pairs_append=int(pairs[app].sum()),
+        flops_append=int(pairs[app].sum()) * 4 * batch.head_dim * batch.num_q_heads,
+        flops=int(pairs.sum()) * 4 * batch.head_dim * batch.num_q_heads,
+    )
+
+
+# ------------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 100 ms in the background."""
+
+    FIELDS = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader",
+                                          "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                c = [x.strip() for x in line.split(",")]
+                if len(c) < 10:
+                    continue
+                if self.uuid and self.uuid not in c[1]:
+                    continue
+                rows.append(c)
+        os.unlink(self.path)
+        if not rows:
+            return None
+
+        def mhz(x):
+            try:
+                return float(x.split()[0])
+            except Exception:
+                return float("nan")
+
+        sm = [mhz(r[2]) for r in rows]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for n, v in zip(names, r[6:10]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mhz(r[3]) for r in rows),
+                "reasons": sorted(reasons), "samples": len(rows)}
+
+
+# ------------------------------------------------------------------ our arm
+
+
+class Stepper:
+    """Device-resident inputs of every layer and one call sequence per step."""
+
+    def __init__(self, batch: W.Batch, dev):
+        from paper_2608_22167_gb300 import mcpu
+
+        self.mcpu = mcpu
+        self.batch = batch
+        self.dev = dev
+        self.sl = torch.from_numpy(batch.seq_lens).to(dev)
+        self.qsl = torch.from_numpy(batch.query_start_loc).to(dev)
+        self.bts = {k: torch.from_numpy(p.block_table).to(dev) for k, p in batch.pools.items()}
+        self.layers = batch.layers
+        lay0 = batch.layers[0]
+        p0 = batch.pools[lay0.pool]
+        self.dims = mcpu.dims(lay0.q, p0.k_cache, self.bts[lay0.pool], self.sl)
+        self.ws = mcpu.new_workspace(self.dims, dev)
+        self.out = torch.empty_like(lay0.q)
+        self.lse = torch.empty(lay0.q.shape[:2], dtype=torch.float32, device=dev)
+        self.launches_per_layer = {}
+        for i, lay in enumerate(batch.layers):
+            cascade = 1 if lay.sliding_window <= 0 else 0
+            self.launches_per_layer[i] = 5 + cascade  # append, plan, [cascade], decode, append-chunk, merge
+
+    def layer_call(self, i, q=None, k_new=None, v_new=None, out=None, lse=None, events=None):
+        m = self.mcpu
+        lay = self.layers[i]
+        pool = self.batch.pools[lay.pool]
+        bt = self.bts[lay.pool]
+        m.mcpu_kv_append(lay.k_new if k_new is None else k_new, lay.v_new if v_new is None else v_new,
+                         pool.k_cache, pool.v_cache, bt, self.sl, self.qsl, m.status_word(self.ws))
+        m.mcpu_paged_attention_forward(lay.q if q is None else q, pool.k_cache, pool.v_cache, bt, self.sl, self.qsl,
+                                       lay.sliding_window, self.batch.softmax_scale,
+                                       self.out if out is None else out, self.lse if lse is None else lse,
+                                       self.ws, phase_events=events)
+
+    def step(self, events=None):
+        for i in range(len(self.layers)):
+            self.layer_call(i, events=None if events is None else events[i])
+
+    @property
+    def launches_per_step(self):
+        return sum(self.launches_per_layer.values())
+
+
+def make_batch(name, dev, rank):
+    fn = W.CONFIGS[name]
+    seed = {"tiny": 1001, "decode": 1002, "mixed": 1003, "long": 1004, "rollout": 1005}[name] + 7 * rank
+    return fn(seed=seed, device=dev)
+
+
+def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int):
+    """Time the oracle on a bounded sample of the workload and scale its
+    throughput to the whole step by attended (query, key) pairs."""
+    import oracle
+
+    rng = np.random.default_rng(seed)
+    L = batch.q_lens
+    dec = np.nonzero(L == 1)[0]
+    app = np.nonzero(L > 1)[0]
+    t_spent = 0.0
+    pairs_done = 0
+    n_tok = 0
+    rounds = 0
+    Wn = batch.layers[0].sliding_window
+    while t_spent < seconds and rounds < 50:
+        rounds += 1
+        rows = list(rng.choice(dec, size=min(6, len(dec)), replace=False)) if len(dec) else []
+        if len(app):
+            rows += list(rng.choice(app, size=min(2, len(app)), replace=False))
+        h = W.host_rows(batch, rows, 0)
+        kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                                  h["seq_lens"], h["query_start_loc"])
+        qsl = h["query_start_loc"]
+        toks = []
+        for i in range(len(h["rows"])):
+            t0, t1 = int(qsl[i]), int(qsl[i + 1])
+            sel = np.arange(t0, t1)
+            if len(sel) > 24:
+                sel = rng.choice(sel, size=24, replace=False)
+            toks += list(sel)
+        toks = np.asarray(toks, np.int64)
+        tk = np.repeat(toks, batch.num_q_heads)
+        hd = np.tile(np.arange(batch.num_q_heads, dtype=np.int32), len(toks))
+        # attended pairs of the sampled queries
+        row_of = np.searchsorted(qsl, toks, side="right") - 1
+        S = h["seq_lens"][row_of].astype(np.int64)
+        Lr = (qsl[row_of + 1] - qsl[row_of]).astype(np.int64)
+        p = S - Lr + (toks - qsl[row_of])
+        vis = p + 1 if Wn <= 0 else np.minimum(p + 1, Wn)
+        t = time.perf_counter()
+        oracle.paged_attention_sampled(h["q"], kc, vc, h["block_table"], h["seq_lens"], qsl, Wn,
+                                       batch.softmax_scale, tk, hd)
+        t_spent += time.perf_counter() - t
+        pairs_done += int(vis.sum()) * batch.num_q_heads
+        n_tok += len(toks)
+    pairs_total = stats_total["pairs"] * batch.num_q_heads
+    est_step_s = t_spent * pairs_total / max(pairs_done, 1)
+    return dict(
+        value=stats_total["kv_bytes"] / est_step_s / 1e9,
+        unit="GB/s",
+        cores=int(oracle.max_threads()),
+        kind="oracle",
+        sample=f"{n_tok} query tokens x {batch.num_q_heads} heads from {rounds} draws of 6 decode + 2 append "
+               f"rows (layer 0), {t_spent:.1f} s of oracle time; step time scaled by attended (query, key) pairs "
+               f"({pairs_done:.3g} of {pairs_total:.3g})",
+        est_step_ms=est_step_s * 1e3,
+        attended_tokens_per_s=stats_total["pairs"] / est_step_s,
+    )
+
+
+def run_ours(args, rank, world, dev):
+    from paper_2608_22167_gb300 import mcpu
+
+    hbm, tc_burst, tc_sust, peak_src = peaks()
+    batch = make_batch(args.workload, dev, rank)
+    st = Stepper(batch, dev)
+    per_layer = [layer_stats(batch, i) for i in range(len(batch.layers))]
+    kv_bytes = sum(s["kv_bytes"] for s in per_layer)
+    pairs = sum(s["pairs"] for s in per_layer)
+
+    # warm-up (also the first call performs the per-device setup)
+    for _ in range(args.warmup):
+        st.step()
+    torch.cuda.synchronize()
+    code, bits = mcpu.mcpu_read_device_status(st.ws)
+    if code != 0:
+        raise RuntimeError(f"device status {bits} after warm-up")
+
+    nl = len(batch.layers)
+    stream = torch.cuda.current_stream()
+    phase = [[[torch.cuda.Event(enable_timing=True) for _ in range(mcpu.NUM_PHASE_EVENTS)] for _ in range(nl)]
+             for _ in range(args.steps)]
+    for s in phase:  # create the events (torch creates them lazily)
+        for lay in s:
+            for e in lay:
+                e.record(stream)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)  # let the sampler start before the timed region
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        starts[k].record(stream)
+        st.step(events=phase[k])
+        ends[k].record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    step_ms = [starts[k].elapsed_time(ends[k]) for k in range(args.steps)]
+    total_ms = float(sum(step_ms))
+    code, bits = mcpu.mcpu_read_device_status(st.ws)
+    if code != 0:
+        raise RuntimeError(f"device status {bits} in the timed region")
+
+    # per-kernel times (ms per launch, averaged over steps and layers of a kind)
+    names = ["plan", "cascade", "decode", "append_chunk", "merge"]
+    ktime = {n: 0.0 for n in names}
+    for k in range(args.steps):
+        for i in range(nl):
+            ev = phase[k][i]
+            for j, n in enumerate(names):
+                ktime[n] += ev[j].elapsed_time(ev[j + 1])
+    ktime = {n: v / args.steps for n, v in ktime.items()}  # ms per step
+    dec_bytes = sum(s["kv_bytes"] - s["kv_bytes_append"] for s in per_layer)
+    app_flops = sum(s["flops_append"] for s in per_layer)
+    dec_ms = ktime["cascade"] + ktime["decode"]
+    app_ms = ktime["append_chunk"]
+    roof_dec = None
+    if dec_ms > 0 and dec_bytes > 0:
+        ach = dec_bytes / (dec_ms * 1e-3) / 1e9
+        roof_dec = {"bound": "hbm", "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
+                    "frac": round(ach / hbm, 4), "traffic": None,
+                    "kernel": "decode_kernel (+cascade pass)", "peak_source": f"{peak_src} hbm_gbs",
+                    "ms_per_step": round(dec_ms, 4)}
+    roof_app = None
+    if app_ms > 0 and app_flops > 0:
+        ach = app_flops / (app_ms * 1e-3) / 1e12
+        roof_app = {"bound": "tensor", "achieved": round(ach, 2), "peak": tc_burst, "unit": "TFLOP/s",
+                    "frac": round(ach / tc_burst, 4), "traffic": None, "kernel": "append_kernel",
+                    "peak_source": f"{peak_src} bf16_tflops (burst)", "ms_per_step": round(app_ms, 4)}
+    cands = [r for r in (roof_dec, roof_app) if r is not None]
+    dominant = max(cands, key=lambda r: r["ms_per_step"]) if cands else None
+
+    # ---- end to end: host buffers, copies inside the timed region
+    lay_host = []
+    for lay in batch.layers:
+        lay_host.append((lay.q.cpu().pin_memory(), lay.k_new.cpu().pin_memory(), lay.v_new.cpu().pin_memory()))
+    meta_host = [torch.from_numpy(batch.seq_lens).pin_memory(), torch.from_numpy(batch.query_start_loc).pin_memory()]
+    bt_host = {k: torch.from_numpy(p.block_table).pin_memory() for k, p in batch.pools.items()}
+    q_d = torch.empty_like(batch.layers[0].q)
+    kn_d = torch.empty_like(batch.layers[0].k_new)
+    vn_d = torch.empty_like(batch.layers[0].v_new)
+    out_h = torch.empty(q_d.shape, dtype=q_d.dtype).pin_memory()
+    lse_h = torch.empty(q_d.shape[:2], dtype=torch.float32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for tr in lay_host for t in tr)
+    h2d += sum(t.numel() * t.element_size() for t in meta_host) + sum(
+        t.numel() * t.element_size() for t in bt_host.values())
+    d2h = (out_h.numel() * out_h.element_size() + lse_h.numel() * 4) * nl
+
+    def e2e_step():
+        st.sl.copy_(meta_host[0], non_blocking=True)
+        st.qsl.copy_(meta_host[1], non_blocking=True)
+        for key, t in bt_host.items():
+            st.bts[key].copy_(t, non_blocking=True)
+        for i in range(nl):
+            qh, knh, vnh = lay_host[i]
+            q_d.copy_(qh, non_blocking=True)
+            kn_d.copy_(knh, non_blocking=True)
+            vn_d.copy_(vnh, non_blocking=True)
+            st.layer_call(i, q=q_d, k_new=kn_d, v_new=vn_d)
+            out_h.copy_(st.out, non_blocking=True)
+            lse_h.copy_(st.lse, non_blocking=True)
+
+    e2e_steps = max(3, min(args.steps, 20))
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+
+    # ---- max over ranks
+    if world > 1:
+        t = torch.tensor([total_ms, e2e_ms], device=dev, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms, e2e_ms = float(t[0]), float(t[1])
+    ms_per_step = total_ms / args.steps
+    value = kv_bytes * world / (ms_per_step * 1e-3) / 1e9
+    e2e_value = kv_bytes * world / (e2e_ms * 1e-3) / 1e9
+
+    res = {
+        "metric": "KV-read HBM GB/s (% of GB300 peak) and attended tokens/s, paged mixed batch",
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V; lengths drawn per the workload recipe)",
+        "config": {
+            "workload": WORKLOAD_DESC[args.workload],
+            "layers": nl,
+            "rows": batch.num_seqs,
+            "query_tokens": batch.total_q,
+            "kv_bytes_per_step": kv_bytes,
+            "attended_pairs_per_step": pairs,
+            "l2": "inputs larger than L2 (KV pool %.1f GB >> 126 MB L2); no flush" % (
+                sum(p.k_cache.numel() * 4 for p in batch.pools.values()) / 1e9),
+            "parallelism": f"replicas x{world} (no exchange step)",
+        },
+        "frac_of_hbm_peak": round(value / world / hbm, 4),
+        "attended_tokens_per_s": round(pairs * world / (ms_per_step * 1e-3), 1),
+        "kernel_ms_per_step": {k: round(v, 4) for k, v in ktime.items()},
+        "roofline": dominant,
+        "roofline_decode": roof_dec,
+        "roofline_append": roof_app,
+        "gpu_launches": st.launches_per_step * args.steps,
+        "e2e": {"value": round(e2e_value, 2), "unit": "GB/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_ms, 4)},
+        "clocks": clocks,
+        "wall_s_timed": round(wall, 3),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        stats0 = per_layer[0]
+        cb = cpu_baseline_sample(batch, {"kv_bytes": stats0["kv_bytes"], "pairs": stats0["pairs"]},
+                                 args.cpu_seconds, seed=99)
+        res["cpu_baseline"] = {k: (round(v, 4) if isinstance(v, float) else v) for k, v in cb.items()}
+    return res
+
+
+def run_reference(args, rank, world):
+    """The oracle (plain CPU definition) timed on the host cores, rank 0 only."""
+    if rank != 0:
+        return None
+    batch = make_batch(args.workload, "cuda" if torch.cuda.is_available() else "cpu", 0)
+    stats0 = layer_stats(batch, 0)
+    nl = len(batch.layers)
+    per_step = max(2.0, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
+    for w in range(args.warmup):
+        cpu_baseline_sample(batch, stats0, per_step / 4, seed=1000 + w)
+    vals, ms = [], []
+    cb = None
+    for k in range(args.steps):
+        cb = cpu_baseline_sample(batch, stats0, per_step, seed=2000 + k)
+        vals.append(cb["value"])
+        ms.append(cb["est_step_ms"] * nl)
+    value = float(statistics.mean(vals))
+    return {
+        "metric": "KV-read HBM GB/s (% of GB300 peak) and attended tokens/s, paged mixed batch",
+        "value": round(value, 4),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(float(statistics.mean(ms)), 2),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V; lengths drawn per the workload recipe)",
+        "config": {"workload": WORKLOAD_DESC[args.workload], "layers": nl, "rows": batch.num_seqs},
+        "impl": "reference",
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cb["cores"], "kind": "oracle",
+                         "sample": cb["sample"]},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(W.CONFIGS), default="mixed")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        torch.distributed.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+
+    if args.impl == "reference":
+        res = run_reference(args, rank, world)
+    else:
+        if not torch.cuda.is_available():
+            raise SystemExit("bench.py needs a CUDA GPU for --impl ours")
+        torch.cuda.set_device(dev)
+        from __graft_entry__ import build
+
+        build()
+        res = run_ours(args, rank, world, dev)
+    if rank == 0 and res is not None:
+        print(json.dumps(res))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

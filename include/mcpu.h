@@ -1,0 +1,162 @@
+/*
+ * mcpu.h -- C ABI of the GB300 (sm_103a) paged-attention hot path.
+ *
+ * The paper (MCP-Universe RL, §3.2) describes a rollout engine that keeps
+ * hundreds of multi-turn tool-use trajectories in flight and notes that the
+ * run stage is bound by GPU generation. Between tool calls every trajectory
+ * either decodes one token or appends a tool-observation chunk, and the n = 8
+ * samples of a GRPO task (§4; App. B, Tab. "hparams") share their prompt.
+ * This library is that generation step's attention: a ragged batch of rows
+ * ("trajectories") whose KV caches live in a paged pool, with
+ *
+ *   mcpu_kv_append                -- writes the new tokens' K/V into their pages
+ *   mcpu_paged_attention_forward  -- causal (optionally sliding-window)
+ *                                    softmax attention of every query token
+ *                                    over its row's paged keys and values,
+ *                                    returning out and the log-sum-exp
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every pointer argument except `dims`/`opts`/`status_bits` is DEVICE
+ *    memory owned by the caller; the library never frees or retains it.
+ *    Tensors are dense, row-major, with the shapes given below. bf16 data and
+ *    the pools must be 16-byte aligned.
+ *  - Work is enqueued on `stream` (NULL = the legacy default stream) and the
+ *    call returns without synchronising. The forward call allocates nothing:
+ *    all scratch lives in the caller's workspace.
+ *  - Host-side argument checks return an error code synchronously and launch
+ *    nothing. Errors only visible on the device (a page id outside the pool,
+ *    L_r > S_r, a wait that timed out) set bits in a status word at the start
+ *    of the workspace and the kernels skip or zero-fill the affected reads;
+ *    read it with mcpu_read_device_status. Nothing traps.
+ *
+ * Notation (row r = one trajectory):
+ *   B  = num_seqs, T = total_q = query_start_loc[B]
+ *   L_r = query_start_loc[r+1] - query_start_loc[r]  (1 for a decode row)
+ *   S_r = seq_lens[r]: KV length of row r AFTER this step's append; the row's
+ *         query tokens occupy positions S_r - L_r .. S_r - 1.
+ *   Query i of row r sits at p = S_r - L_r + i and sees key j iff j <= p and,
+ *   when sliding_window W > 0, p - j < W. q head h reads kv head h / (H_q/H_kv).
+ *
+ * Layouts:
+ *   q             [T, H_q, D]          bf16
+ *   k_new, v_new  [T, H_kv, D]         bf16  (one row per query token)
+ *   k_cache, v_cache [num_pages, H_kv, page_size, D] bf16: the (page, kv head)
+ *                 block is page_size * D * 2 contiguous bytes.
+ *   block_table   [B, max_pages_per_seq] int32: logical page -> physical page.
+ *                 Entries no query can see may hold anything (e.g. -1).
+ *   seq_lens      [B] int32;  query_start_loc [B + 1] int32 (prefix sums, [0] = 0)
+ *   out           [T, H_q, D] bf16;  lse [T, H_q] float (natural log of the
+ *                 softmax normaliser sum_j exp(scale * q.k_j); -inf if empty)
+ *
+ * Supported now: D = 64, page_size = 16, H_q / H_kv in {1, 2, 4, 8},
+ * num_seqs <= 4096. Anything else returns MCPU_ERR_UNSUPPORTED.
+ */
+#ifndef MCPU_H
+#define MCPU_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t (a CUstream_st pointer). */
+typedef struct CUstream_st* mcpu_stream_t;
+
+typedef enum mcpu_status {
+  MCPU_OK = 0,
+  MCPU_ERR_INVALID_ARG = 1,          /* null/misaligned pointer, inconsistent dims */
+  MCPU_ERR_UNSUPPORTED = 2,          /* valid but not implemented (D, page size, ratio) */
+  MCPU_ERR_WORKSPACE_TOO_SMALL = 3,  /* workspace_bytes < mcpu_workspace_size(dims) */
+  MCPU_ERR_CUDA = 4,                 /* a CUDA runtime call failed (launch, attributes) */
+  MCPU_ERR_BAD_PAGE = 5,             /* device: a needed block-table entry is outside the pool */
+  MCPU_ERR_BAD_LENGTHS = 6,          /* device: L_r > S_r, L_r < 0, S_r beyond the table, or
+                                        query_start_loc[0] != 0 / [B] != total_q */
+  MCPU_ERR_TIMEOUT = 7,              /* device: a bounded wait gave up */
+  MCPU_ERR_INTERNAL = 8              /* device: work plan overflowed its bound */
+} mcpu_status;
+
+typedef struct mcpu_dims {
+  int32_t num_seqs;           /* B */
+  int32_t total_q;            /* T = query_start_loc[B] */
+  int32_t max_pages_per_seq;  /* columns of block_table */
+  int32_t num_pages;          /* physical pages in each of k_cache / v_cache */
+  int32_t num_q_heads;        /* H_q */
+  int32_t num_kv_heads;       /* H_kv */
+  int32_t head_dim;           /* D (64) */
+  int32_t page_size;          /* tokens per page (16) */
+} mcpu_dims;
+
+/* Optional knobs of the forward pass; pass NULL for the defaults. */
+#define MCPU_FLAG_NO_CASCADE 0x1u   /* never run the shared-prefix (cascade) pass */
+typedef struct mcpu_options {
+  uint32_t flags;             /* MCPU_FLAG_* */
+  int32_t split_pages;        /* > 0: KV split length of decode rows, in pages (0 = auto) */
+  /* Optional timing hook: if non-NULL, MCPU_NUM_PHASE_EVENTS cudaEvent_t
+   * handles (created by the caller) that the call records on `stream`:
+   * [0] before the planner, [1] after it, [2] after the cascade pass,
+   * [3] after split-KV decode, [4] after the append-chunk kernel,
+   * [5] after the merge. Differences of consecutive events time each kernel. */
+  void* const* phase_events;
+} mcpu_options;
+#define MCPU_NUM_PHASE_EVENTS 6
+
+/* Bytes of workspace mcpu_paged_attention_forward needs for these dims
+ * (depends on num_seqs, total_q and the head counts only). 0 if dims are
+ * invalid. The first 4 bytes are the device status word: zero the workspace
+ * once before first use (or call mcpu_reset_device_status). */
+size_t mcpu_workspace_size(const mcpu_dims* dims);
+
+/*
+ * KV append (the new tokens of every row enter the cache).
+ * For each row r and i < L_r, copies k_new[query_start_loc[r] + i] (all kv
+ * heads) bit for bit to k_cache[block_table[r][pos / page]][h][pos % page]
+ * with pos = S_r - L_r + i; likewise v_new into v_cache. Decode rows append
+ * their one token; append rows their whole chunk. Nothing else is written.
+ * `status_word` (device int32, may be the workspace start) receives
+ * device-side error bits; a row with an invalid page or length is skipped.
+ */
+mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                           const int32_t* block_table, const int32_t* seq_lens,
+                           const int32_t* query_start_loc, const mcpu_dims* dims,
+                           int32_t* status_word, mcpu_stream_t stream);
+
+/*
+ * Paged attention forward over a mixed batch of decode rows (L_r = 1) and
+ * append rows (L_r > 1, causal within the chunk), with an optional sliding
+ * window (W <= 0: full context). Rows with L_r = 0 produce nothing.
+ * softmax_scale multiplies q.k (1/sqrt(D) for gpt-oss). Rows that are
+ * adjacent in the batch and whose block tables start with the same physical
+ * pages (a GRPO group's shared prompt) are detected on the device and their
+ * common full pages are read once for the whole group (full-context calls
+ * only). Long decode rows are split over SMs and merged by log-sum-exp.
+ * Results do not depend on the split or cascade choices beyond rounding.
+ */
+mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, const void* v_cache,
+                                         const int32_t* block_table, const int32_t* seq_lens,
+                                         const int32_t* query_start_loc, int32_t sliding_window,
+                                         float softmax_scale, const mcpu_dims* dims, void* out,
+                                         float* lse, void* workspace, size_t workspace_bytes,
+                                         const mcpu_options* opts, mcpu_stream_t stream);
+
+/* Synchronises `stream`, reads the workspace status word and maps it to the
+ * most severe mcpu_status (MCPU_OK if clear). The raw bits go to
+ * *status_bits if non-NULL. The word is not cleared. */
+mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream, int32_t* status_bits);
+
+/* Enqueues a clear of the workspace status word on `stream`. */
+mcpu_status mcpu_reset_device_status(void* workspace, mcpu_stream_t stream);
+
+/* Static, human-readable name of a status code. */
+const char* mcpu_status_string(mcpu_status status);
+
+/* Version of this ABI (bumped on any signature change). */
+int32_t mcpu_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MCPU_H */

@@ -1,0 +1,245 @@
+// C ABI of the paged-attention path (declared in include/mcpu.h): host-side
+// argument checks, per-device one-time setup (kernel attributes, occupancy),
+// TMA descriptors of the two KV pools, and the launch sequence
+//   planner -> cascade pass -> split-KV decode -> append-chunk -> LSE merge
+// on the caller's stream. Nothing here allocates device memory.
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "../../include/mcpu.h"
+#include "common.cuh"
+
+namespace mcpu {
+cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream);
+cudaError_t prepare_plan_kernel();
+cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
+                          bool cascade, cudaStream_t stream);
+cudaError_t prepare_decode_kernels(int* bpsm_decode, int* bpsm_cascade);
+cudaError_t launch_append(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
+                          cudaStream_t stream);
+cudaError_t prepare_append_kernel(int* bpsm);
+cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                             const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
+                             int32_t* status, int32_t num_seqs, int32_t total_q, int32_t max_pages,
+                             int32_t num_pages, int32_t num_kv_heads, cudaStream_t stream);
+}  // namespace mcpu
+
+namespace {
+
+using namespace mcpu;
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+  bool ready = false;
+  int sms = 0;
+  int bpsm_decode = 0, bpsm_cascade = 0, bpsm_append = 0;
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+mcpu_status device_state(DeviceState** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MCPU_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mu);
+  DeviceState& st = g_dev[dev];
+  if (!st.ready) {
+    if (!g_encode) {
+      void* fn = nullptr;
+      cudaDriverEntryPointQueryResult q;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return MCPU_ERR_CUDA;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    if (cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (prepare_plan_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
+    if (prepare_decode_kernels(&st.bpsm_decode, &st.bpsm_cascade) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (prepare_append_kernel(&st.bpsm_append) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1) return MCPU_ERR_CUDA;
+    st.ready = true;
+  }
+  *out = &st;
+  return MCPU_OK;
+}
+
+// 2-D view of a pool: rows of D = 64 bf16 (128 bytes), num_pages*H_kv*16 rows;
+// boxes of one (page, kv head) block = 16 rows, 128-byte swizzle.
+bool encode_pool(CUtensorMap* map, const void* pool, int64_t rows) {
+  cuuint64_t dims[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)kRowBytes};
+  cuuint32_t box[2] = {(cuuint32_t)kHeadDim, (cuuint32_t)kPage};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(pool), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Checks shared by both entry points. Returns MCPU_OK or the error.
+mcpu_status check_dims(const mcpu_dims* d) {
+  if (!d) return MCPU_ERR_INVALID_ARG;
+  if (d->num_seqs < 0 || d->total_q < 0 || d->max_pages_per_seq < 0 || d->num_pages < 0 || d->num_q_heads <= 0 ||
+      d->num_kv_heads <= 0 || d->head_dim <= 0 || d->page_size <= 0)
+    return MCPU_ERR_INVALID_ARG;
+  if (d->num_q_heads % d->num_kv_heads != 0) return MCPU_ERR_INVALID_ARG;
+  if (d->head_dim != kHeadDim || d->page_size != kPage) return MCPU_ERR_UNSUPPORTED;
+  const int g = d->num_q_heads / d->num_kv_heads;
+  if (g != 1 && g != 2 && g != 4 && g != 8) return MCPU_ERR_UNSUPPORTED;
+  if (d->num_seqs > kMaxSeqs) return MCPU_ERR_UNSUPPORTED;
+  // pool rows must stay addressable by 32-bit TMA coordinates
+  if ((int64_t)d->num_pages * d->num_kv_heads * kPage >= (int64_t)0x7fff0000) return MCPU_ERR_UNSUPPORTED;
+  if ((int64_t)d->max_pages_per_seq * kPage >= (int64_t)0x7fff0000) return MCPU_ERR_UNSUPPORTED;
+  return MCPU_OK;
+}
+
+mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : MCPU_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t mcpu_abi_version(void) { return 1; }
+
+const char* mcpu_status_string(mcpu_status s) {
+  switch (s) {
+    case MCPU_OK: return "ok";
+    case MCPU_ERR_INVALID_ARG: return "invalid argument";
+    case MCPU_ERR_UNSUPPORTED: return "unsupported configuration";
+    case MCPU_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case MCPU_ERR_CUDA: return "CUDA runtime error";
+    case MCPU_ERR_BAD_PAGE: return "block table names a page outside the pool";
+    case MCPU_ERR_BAD_LENGTHS: return "inconsistent seq_lens / query_start_loc";
+    case MCPU_ERR_TIMEOUT: return "device wait timed out";
+    case MCPU_ERR_INTERNAL: return "work plan exceeded its bound";
+  }
+  return "unknown status";
+}
+
+size_t mcpu_workspace_size(const mcpu_dims* dims) {
+  if (check_dims(dims) != MCPU_OK) return 0;
+  const int g = dims->num_q_heads / dims->num_kv_heads;
+  return workspace_layout(dims->num_seqs, dims->total_q, dims->num_q_heads, g).total;
+}
+
+mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                           const int32_t* block_table, const int32_t* seq_lens, const int32_t* query_start_loc,
+                           const mcpu_dims* dims, int32_t* status_word, mcpu_stream_t stream) {
+  mcpu_status st = check_dims(dims);
+  if (st != MCPU_OK) return st;
+  if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
+  if (!k_new || !v_new || !k_cache || !v_cache || !block_table || !seq_lens || !query_start_loc || !status_word)
+    return MCPU_ERR_INVALID_ARG;
+  if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) ||
+      !aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(query_start_loc, 4) || !aligned(status_word, 4))
+    return MCPU_ERR_INVALID_ARG;
+  if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  return from_cuda(launch_kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start_loc,
+                                    status_word, dims->num_seqs, dims->total_q, dims->max_pages_per_seq,
+                                    dims->num_pages, dims->num_kv_heads, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, const void* v_cache,
+                                         const int32_t* block_table, const int32_t* seq_lens,
+                                         const int32_t* query_start_loc, int32_t sliding_window, float softmax_scale,
+                                         const mcpu_dims* dims, void* out, float* lse, void* workspace,
+                                         size_t workspace_bytes, const mcpu_options* opts, mcpu_stream_t stream) {
+  mcpu_status st = check_dims(dims);
+  if (st != MCPU_OK) return st;
+  if (!(softmax_scale == softmax_scale) || softmax_scale > 3.0e38f || softmax_scale < -3.0e38f)
+    return MCPU_ERR_INVALID_ARG;
+  if (!workspace) return MCPU_ERR_INVALID_ARG;
+  if (workspace_bytes < mcpu_workspace_size(dims)) return MCPU_ERR_WORKSPACE_TOO_SMALL;
+  if (!aligned(workspace, 256)) return MCPU_ERR_INVALID_ARG;
+  if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
+  if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !query_start_loc || !out || !lse)
+    return MCPU_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(lse, 4) ||
+      !aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(query_start_loc, 4))
+    return MCPU_ERR_INVALID_ARG;
+  if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  if (opts && opts->split_pages < 0) return MCPU_ERR_INVALID_ARG;
+
+  DeviceState* dev = nullptr;
+  st = device_state(&dev);
+  if (st != MCPU_OK) return st;
+
+  const int64_t rows = (int64_t)dims->num_pages * dims->num_kv_heads * kPage;
+  CUtensorMap kmap, vmap;
+  if (!encode_pool(&kmap, k_cache, rows) || !encode_pool(&vmap, v_cache, rows)) return MCPU_ERR_INVALID_ARG;
+
+  AttnParams p;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.block_table = block_table;
+  p.seq_lens = seq_lens;
+  p.qsl = query_start_loc;
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.lse = lse;
+  p.ws = static_cast<uint8_t*>(workspace);
+  p.num_seqs = dims->num_seqs;
+  p.total_q = dims->total_q;
+  p.max_pages = dims->max_pages_per_seq;
+  p.num_pages = dims->num_pages;
+  p.num_q_heads = dims->num_q_heads;
+  p.num_kv_heads = dims->num_kv_heads;
+  p.group = dims->num_q_heads / dims->num_kv_heads;
+  p.lay = workspace_layout(p.num_seqs, p.total_q, p.num_q_heads, p.group);
+  p.window = sliding_window > 0 ? sliding_window : 0;
+  p.scale_log2 = softmax_scale * 1.4426950408889634f;
+  p.total_warps_hint = dev->sms * dev->bpsm_decode * 4;
+  p.forced_split_pages = opts ? opts->split_pages : 0;
+  p.cascade_enabled = (opts && (opts->flags & MCPU_FLAG_NO_CASCADE)) ? 0 : 1;
+  p.oob_row = (int32_t)rows;
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  void* const* ev = opts ? opts->phase_events : nullptr;
+  auto mark = [&](int i) -> cudaError_t {
+    return ev ? cudaEventRecord(reinterpret_cast<cudaEvent_t>(ev[i]), s) : cudaSuccess;
+  };
+  cudaError_t e = mark(0);
+  if (e == cudaSuccess) e = launch_plan(p, s);
+  if (e == cudaSuccess) e = mark(1);
+  if (e == cudaSuccess && p.cascade_enabled && p.window == 0)
+    e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, s);
+  if (e == cudaSuccess) e = mark(2);
+  if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s);
+  if (e == cudaSuccess) e = mark(3);
+  if (e == cudaSuccess) e = launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
+  if (e == cudaSuccess) e = mark(4);
+  if (e == cudaSuccess) {
+    const int want = (p.num_seqs * p.num_q_heads + 7) / 8;
+    const int grid = want < dev->sms * 8 ? (want > 0 ? want : 1) : dev->sms * 8;
+    e = launch_merge(p, grid, s);
+  }
+  if (e == cudaSuccess) e = mark(5);
+  return from_cuda(e);
+}
+
+mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream, int32_t* status_bits) {
+  if (!workspace) return MCPU_ERR_INVALID_ARG;
+  int32_t bits = 0;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&bits, workspace, sizeof(bits), cudaMemcpyDeviceToHost, s) != cudaSuccess) return MCPU_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return MCPU_ERR_CUDA;
+  if (status_bits) *status_bits = bits;
+  if (bits & kStatusTimeout) return MCPU_ERR_TIMEOUT;
+  if (bits & kStatusBadPage) return MCPU_ERR_BAD_PAGE;
+  if (bits & kStatusBadLengths) return MCPU_ERR_BAD_LENGTHS;
+  if (bits & kStatusPlanOverflow) return MCPU_ERR_INTERNAL;
+  return MCPU_OK;
+}
+
+mcpu_status mcpu_reset_device_status(void* workspace, mcpu_stream_t stream) {
+  if (!workspace) return MCPU_ERR_INVALID_ARG;
+  return from_cuda(cudaMemsetAsync(workspace, 0, sizeof(int32_t), reinterpret_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

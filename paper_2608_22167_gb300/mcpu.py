@@ -1,0 +1,199 @@
+"""Thin ctypes binding of libmcpu.so (include/mcpu.h).
+
+Argument marshalling only: every function forwards device pointers of torch
+tensors, the sizes read from their shapes and the current CUDA stream to the
+C entry point of the same name, and raises ``McpuError`` on a non-OK status.
+No computation happens here and there is no fallback: if the library is
+missing, importing this module fails.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_build", "libmcpu.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(
+        f"libmcpu.so not found at {LIB_PATH}; build it first with "
+        "`python -c 'import __graft_entry__ as g; g.build()'` (needs nvcc)"
+    )
+_lib = ctypes.CDLL(LIB_PATH)
+
+STATUS = {
+    0: "MCPU_OK",
+    1: "MCPU_ERR_INVALID_ARG",
+    2: "MCPU_ERR_UNSUPPORTED",
+    3: "MCPU_ERR_WORKSPACE_TOO_SMALL",
+    4: "MCPU_ERR_CUDA",
+    5: "MCPU_ERR_BAD_PAGE",
+    6: "MCPU_ERR_BAD_LENGTHS",
+    7: "MCPU_ERR_TIMEOUT",
+    8: "MCPU_ERR_INTERNAL",
+}
+FLAG_NO_CASCADE = 0x1
+
+# Device status bits (first word of the workspace).
+STATUS_BAD_PAGE = 1
+STATUS_BAD_LENGTHS = 2
+STATUS_TIMEOUT = 4
+STATUS_PLAN_OVERFLOW = 8
+
+
+class McpuError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        name = STATUS.get(code, str(code))
+        msg = _lib.mcpu_status_string(code).decode()
+        super().__init__(f"{where}: {name} ({msg})")
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [
+        ("num_seqs", ctypes.c_int32),
+        ("total_q", ctypes.c_int32),
+        ("max_pages_per_seq", ctypes.c_int32),
+        ("num_pages", ctypes.c_int32),
+        ("num_q_heads", ctypes.c_int32),
+        ("num_kv_heads", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32),
+        ("page_size", ctypes.c_int32),
+    ]
+
+
+class Options(ctypes.Structure):
+    _fields_ = [("flags", ctypes.c_uint32), ("split_pages", ctypes.c_int32), ("phase_events", ctypes.c_void_p)]
+
+
+NUM_PHASE_EVENTS = 6
+
+
+_P = ctypes.c_void_p
+_lib.mcpu_workspace_size.argtypes = [ctypes.POINTER(Dims)]
+_lib.mcpu_workspace_size.restype = ctypes.c_size_t
+_lib.mcpu_kv_append.argtypes = [_P, _P, _P, _P, _P, _P, _P, ctypes.POINTER(Dims), _P, _P]
+_lib.mcpu_kv_append.restype = ctypes.c_int
+_lib.mcpu_paged_attention_forward.argtypes = [
+    _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P, ctypes.c_size_t,
+    ctypes.POINTER(Options), _P,
+]
+_lib.mcpu_paged_attention_forward.restype = ctypes.c_int
+_lib.mcpu_read_device_status.argtypes = [_P, _P, ctypes.POINTER(ctypes.c_int32)]
+_lib.mcpu_read_device_status.restype = ctypes.c_int
+_lib.mcpu_reset_device_status.argtypes = [_P, _P]
+_lib.mcpu_reset_device_status.restype = ctypes.c_int
+_lib.mcpu_status_string.argtypes = [ctypes.c_int]
+_lib.mcpu_status_string.restype = ctypes.c_char_p
+_lib.mcpu_abi_version.argtypes = []
+_lib.mcpu_abi_version.restype = ctypes.c_int32
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(code, where):
+    if code != 0:
+        raise McpuError(code, where)
+
+
+def dims(q, k_cache, block_table, seq_lens) -> Dims:
+    """mcpu_dims from tensor shapes: q [T, Hq, D], k_cache [P, Hkv, page, D],
+    block_table [B, max_pages], seq_lens [B]."""
+    return Dims(
+        num_seqs=int(seq_lens.shape[0]),
+        total_q=int(q.shape[0]),
+        max_pages_per_seq=int(block_table.shape[1]),
+        num_pages=int(k_cache.shape[0]),
+        num_q_heads=int(q.shape[1]),
+        num_kv_heads=int(k_cache.shape[1]),
+        head_dim=int(q.shape[2]),
+        page_size=int(k_cache.shape[2]),
+    )
+
+
+def mcpu_abi_version() -> int:
+    return int(_lib.mcpu_abi_version())
+
+
+def mcpu_status_string(code: int) -> str:
+    return _lib.mcpu_status_string(code).decode()
+
+
+def mcpu_workspace_size(d: Dims) -> int:
+    return int(_lib.mcpu_workspace_size(ctypes.byref(d)))
+
+
+def mcpu_kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start_loc, status_word,
+                   stream=None):
+    """status_word: a device int32 tensor (e.g. ``workspace[:4].view(torch.int32)``)."""
+    d = Dims(
+        num_seqs=int(seq_lens.shape[0]),
+        total_q=int(k_new.shape[0]),
+        max_pages_per_seq=int(block_table.shape[1]),
+        num_pages=int(k_cache.shape[0]),
+        num_q_heads=int(k_cache.shape[1]),
+        num_kv_heads=int(k_cache.shape[1]),
+        head_dim=int(k_cache.shape[3]),
+        page_size=int(k_cache.shape[2]),
+    )
+    _check(
+        _lib.mcpu_kv_append(_ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(block_table),
+                            _ptr(seq_lens), _ptr(query_start_loc), ctypes.byref(d), _ptr(status_word),
+                            _stream(stream)),
+        "mcpu_kv_append",
+    )
+
+
+def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, sliding_window,
+                                 softmax_scale, out, lse, workspace, flags=0, split_pages=0, stream=None,
+                                 phase_events=None):
+    """phase_events: optional list of NUM_PHASE_EVENTS torch.cuda.Event the
+    call records around its kernels (see mcpu_options in include/mcpu.h)."""
+    d = dims(q, k_cache, block_table, seq_lens)
+    opts = Options(flags=int(flags), split_pages=int(split_pages), phase_events=None)
+    if phase_events is not None:
+        assert len(phase_events) == NUM_PHASE_EVENTS
+        arr = (ctypes.c_void_p * NUM_PHASE_EVENTS)(*[ctypes.c_void_p(e.cuda_event) for e in phase_events])
+        opts.phase_events = ctypes.cast(arr, ctypes.c_void_p)
+    _check(
+        _lib.mcpu_paged_attention_forward(
+            _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc),
+            int(sliding_window), float(softmax_scale), ctypes.byref(d), _ptr(out), _ptr(lse), _ptr(workspace),
+            int(workspace.numel() * workspace.element_size()), ctypes.byref(opts), _stream(stream),
+        ),
+        "mcpu_paged_attention_forward",
+    )
+
+
+def mcpu_read_device_status(workspace, stream=None):
+    """(mcpu status code, raw status bits) of the workspace's status word."""
+    bits = ctypes.c_int32(0)
+    code = _lib.mcpu_read_device_status(_ptr(workspace), _stream(stream), ctypes.byref(bits))
+    return int(code), int(bits.value)
+
+
+def mcpu_reset_device_status(workspace, stream=None):
+    _check(_lib.mcpu_reset_device_status(_ptr(workspace), _stream(stream)), "mcpu_reset_device_status")
+
+
+def new_workspace(d: Dims, device="cuda") -> torch.Tensor:
+    """A zeroed workspace of the size mcpu_workspace_size(d) asks for."""
+    n = mcpu_workspace_size(d)
+    if n == 0:
+        raise McpuError(1, "mcpu_workspace_size")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def status_word(workspace) -> torch.Tensor:
+    """The device int32 status word at the start of a workspace."""
+    return workspace[:4].view(torch.int32)

@@ -1,0 +1,118 @@
+"""Helpers shared by the GPU tests: run a batch through the C ABI and
+compare with the oracle at the stated tolerances.
+
+Tolerances (floating point): out max |gpu - oracle| <= 2e-2 and
+max |gpu - oracle| / max |oracle| <= 1e-2 per checked set (elementwise
+relative error is meaningless for outputs near zero: long-context outputs are
+averages of many N(0,1) rows), lse max abs <= 1e-3. KV append: bit-exact.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+import workloads as W
+from paper_2608_22167_gb300 import mcpu
+
+OUT_ABS = 2e-2
+OUT_REL = 1e-2
+LSE_ABS = 1e-3
+
+
+class Run:
+    """Device copies of one layer of a batch plus the outputs of one call."""
+
+    def __init__(self, batch: W.Batch, layer: int = 0, device="cuda"):
+        self.batch = batch
+        self.layer = layer
+        lay = batch.layers[layer]
+        pool = batch.pools[lay.pool]
+        dev = torch.device(device)
+        self.q = lay.q.to(dev)
+        self.k_new = lay.k_new.to(dev)
+        self.v_new = lay.v_new.to(dev)
+        self.kc = pool.k_cache.to(dev)
+        self.vc = pool.v_cache.to(dev)
+        if self.kc.data_ptr() == pool.k_cache.data_ptr():  # already on the device: keep the input intact
+            self.kc = self.kc.clone()
+            self.vc = self.vc.clone()
+        self.bt = torch.from_numpy(pool.block_table).to(dev)
+        self.sl = torch.from_numpy(batch.seq_lens).to(dev)
+        self.qsl = torch.from_numpy(batch.query_start_loc).to(dev)
+        self.window = lay.sliding_window
+        self.dims = mcpu.dims(self.q, self.kc, self.bt, self.sl)
+        self.ws = mcpu.new_workspace(self.dims, dev)
+        self.out = torch.full_like(self.q, float("nan"))
+        self.lse = torch.full(self.q.shape[:2], float("nan"), dtype=torch.float32, device=dev)
+
+    def append(self):
+        mcpu.mcpu_kv_append(self.k_new, self.v_new, self.kc, self.vc, self.bt, self.sl, self.qsl,
+                            mcpu.status_word(self.ws))
+
+    def forward(self, flags=0, split_pages=0):
+        mcpu.mcpu_paged_attention_forward(self.q, self.kc, self.vc, self.bt, self.sl, self.qsl, self.window,
+                                          self.batch.softmax_scale, self.out, self.lse, self.ws, flags=flags,
+                                          split_pages=split_pages)
+
+    def status(self):
+        return mcpu.mcpu_read_device_status(self.ws)
+
+    def header(self):
+        h = self.ws[:32].view(torch.int32).cpu().numpy()
+        return dict(status=int(h[0]), n_decode=int(h[1]), n_cascade=int(h[2]), n_append=int(h[3]),
+                    n_merge=int(h[4]), split_pages=int(h[5]), n_parts=int(h[6]))
+
+    def out_host(self):
+        return self.out.float().cpu().numpy(), self.lse.cpu().numpy()
+
+
+def oracle_full(batch: W.Batch, layer: int = 0):
+    """Oracle outputs of a whole (small) layer, append applied first."""
+    h = W.host_inputs(batch, layer)
+    kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                              h["seq_lens"], h["query_start_loc"])
+    out, lse = oracle.paged_attention(h["q"], kc, vc, h["block_table"], h["seq_lens"], h["query_start_loc"],
+                                      h["sliding_window"], h["softmax_scale"])
+    return oracle.bf16_bits_to_float(out), lse, (kc, vc)
+
+
+def oracle_sampled(batch: W.Batch, rows, n_per_row: int, rng, layer: int = 0):
+    """Oracle at sampled (token, head) pairs of the given rows: returns
+    (token indices in the batch, heads, out [n, D], lse [n])."""
+    h = W.host_rows(batch, rows, layer)
+    kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                              h["seq_lens"], h["query_start_loc"])
+    qsl = h["query_start_loc"]
+    toks, heads = [], []
+    for i in range(len(h["rows"])):
+        t0, t1 = int(qsl[i]), int(qsl[i + 1])
+        if t1 == t0:
+            continue
+        # always the first and last token of the row, then random ones
+        cand = [t0, t1 - 1] + list(rng.integers(t0, t1, size=max(0, n_per_row - 2)))
+        for t in cand[:n_per_row]:
+            toks.append(int(t))
+            heads.append(int(rng.integers(0, batch.num_q_heads)))
+    toks = np.asarray(toks, np.int64)
+    heads = np.asarray(heads, np.int32)
+    out, lse = oracle.paged_attention_sampled(h["q"], kc, vc, h["block_table"], h["seq_lens"], qsl,
+                                              h["sliding_window"], h["softmax_scale"], toks, heads)
+    return h["token_map"][toks], heads, oracle.bf16_bits_to_float(out), lse
+
+
+def assert_parity(got_out, got_lse, ref_out, ref_lse, what=""):
+    got_out = np.asarray(got_out, np.float64)
+    ref_out = np.asarray(ref_out, np.float64)
+    assert np.all(np.isfinite(got_out)), f"{what}: non-finite outputs"
+    err = np.abs(got_out - ref_out)
+    max_abs = float(err.max()) if err.size else 0.0
+    scale = float(np.abs(ref_out).max()) if err.size else 1.0
+    rel = max_abs / max(scale, 1e-30)
+    fin = np.isfinite(ref_lse)
+    assert np.array_equal(fin, np.isfinite(got_lse)), f"{what}: lse finiteness differs"
+    lse_err = float(np.abs(np.asarray(got_lse)[fin] - ref_lse[fin]).max()) if fin.any() else 0.0
+    assert max_abs <= OUT_ABS, f"{what}: max abs err {max_abs:.3e}"
+    assert rel <= OUT_REL, f"{what}: norm-relative err {rel:.3e}"
+    assert lse_err <= LSE_ABS, f"{what}: lse abs err {lse_err:.3e}"
+    return max_abs, rel, lse_err

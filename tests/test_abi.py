@@ -1,0 +1,138 @@
+"""The C ABI library loads, exports every function include/mcpu.h declares,
+and rejects bad arguments on the host before touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_22167_gb300 import build
+
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "mcpu.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(mcpu_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_two_hot_path_calls():
+    names = _declared_functions()
+    assert "mcpu_kv_append" in names and "mcpu_paged_attention_forward" in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in _declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_binding_uses_the_same_names():
+    from paper_2608_22167_gb300 import mcpu
+
+    for name in _declared_functions():
+        assert hasattr(mcpu, name), name
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("num_seqs", "total_q", "max_pages_per_seq", "num_pages",
+                                              "num_q_heads", "num_kv_heads", "head_dim", "page_size")]
+
+
+def _fn(lib, name):
+    f = getattr(lib, name)
+    f.restype = ctypes.c_int
+    return f
+
+
+def test_workspace_size(lib):
+    lib.mcpu_workspace_size.restype = ctypes.c_size_t
+    ok = Dims(4, 4, 19, 34, 8, 2, 64, 16)
+    n = lib.mcpu_workspace_size(ctypes.byref(ok))
+    assert n > 0 and n % 256 == 0
+    bigger = Dims(400, 40000, 19, 34, 8, 2, 64, 16)
+    assert lib.mcpu_workspace_size(ctypes.byref(bigger)) > n
+    for bad in (Dims(4, 4, 19, 34, 8, 3, 64, 16),     # H_q not a multiple of H_kv
+                Dims(4, 4, 19, 34, 8, 2, 128, 16),    # head_dim unsupported
+                Dims(4, 4, 19, 34, 8, 2, 64, 32),     # page size unsupported
+                Dims(4, 4, 19, 34, 48, 2, 64, 16),    # group 24 unsupported
+                Dims(5000, 4, 19, 34, 8, 2, 64, 16),  # too many rows
+                Dims(-1, 4, 19, 34, 8, 2, 64, 16)):
+        assert lib.mcpu_workspace_size(ctypes.byref(bad)) == 0
+    assert lib.mcpu_workspace_size(None) == 0
+
+
+def test_host_validation_errors(lib):
+    fwd = _fn(lib, "mcpu_paged_attention_forward")
+    fwd.argtypes = [ctypes.c_void_p] * 6 + [ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims)] + \
+        [ctypes.c_void_p] * 3 + [ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]
+    d = Dims(4, 4, 19, 34, 8, 2, 64, 16)
+    P = 1 << 20  # a 256-byte-aligned fake address: never dereferenced by these calls
+    lib.mcpu_workspace_size.restype = ctypes.c_size_t
+    need = lib.mcpu_workspace_size(ctypes.byref(d))
+    args = [P] * 6 + [0, 0.125, ctypes.byref(d), P, P, P, need, None, None]
+    # dims NULL
+    a = list(args); a[8] = None
+    assert fwd(*a) == 1
+    # workspace too small
+    a = list(args); a[12] = need - 1
+    assert fwd(*a) == 3
+    # misaligned workspace
+    a = list(args); a[11] = P + 8
+    assert fwd(*a) == 1
+    # NaN scale
+    a = list(args); a[7] = float("nan")
+    assert fwd(*a) == 1
+    # unsupported head dim
+    d2 = Dims(4, 4, 19, 34, 8, 2, 128, 16)
+    a = list(args); a[8] = ctypes.byref(d2)
+    assert fwd(*a) == 2
+    # misaligned q (needs 16 bytes)
+    a = list(args); a[0] = P + 2
+    assert fwd(*a) == 1
+    # null output
+    a = list(args); a[9] = None
+    assert fwd(*a) == 1
+    # empty batch: nothing to do, no launch, OK
+    d3 = Dims(0, 0, 19, 34, 8, 2, 64, 16)
+    a = list(args); a[8] = ctypes.byref(d3); a[12] = lib.mcpu_workspace_size(ctypes.byref(d3))
+    assert fwd(*a) == 0
+
+
+def test_kv_append_host_validation(lib):
+    app = _fn(lib, "mcpu_kv_append")
+    app.argtypes = [ctypes.c_void_p] * 7 + [ctypes.POINTER(Dims), ctypes.c_void_p, ctypes.c_void_p]
+    d = Dims(4, 4, 19, 34, 2, 2, 64, 16)
+    P = 1 << 20
+    assert app(P, P, P, P, P, P, P, ctypes.byref(d), None, None) == 1      # no status word
+    assert app(P + 4, P, P, P, P, P, P, ctypes.byref(d), P, None) == 1     # misaligned k_new
+    d0 = Dims(0, 0, 19, 34, 2, 2, 64, 16)
+    assert app(P, P, P, P, P, P, P, ctypes.byref(d0), P, None) == 0        # empty: no-op
+
+
+def test_status_strings(lib):
+    lib.mcpu_status_string.restype = ctypes.c_char_p
+    seen = set()
+    for code in range(9):
+        s = lib.mcpu_status_string(code)
+        assert s and s not in seen
+        seen.add(s)
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-GPU error path")
+def test_no_gpu_is_a_clean_error(lib):
+    fwd = _fn(lib, "mcpu_paged_attention_forward")
+    fwd.argtypes = [ctypes.c_void_p] * 6 + [ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims)] + \
+        [ctypes.c_void_p] * 3 + [ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]
+    d = Dims(4, 4, 19, 34, 8, 2, 64, 16)
+    lib.mcpu_workspace_size.restype = ctypes.c_size_t
+    need = lib.mcpu_workspace_size(ctypes.byref(d))
+    P = 1 << 20
+    assert fwd(P, P, P, P, P, P, 0, 0.125, ctypes.byref(d), P, P, P, need, None, None) == 4

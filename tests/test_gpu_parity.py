@@ -1,0 +1,181 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle on the
+same seeded inputs, element by element on small batches and on sampled
+outputs at the full workload sizes. KV append is compared bit for bit."""
+import numpy as np
+import pytest
+import torch
+
+import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    from _gpu import Run, assert_parity, oracle_full, oracle_sampled
+    from paper_2608_22167_gb300 import mcpu
+
+
+def _full_check(batch, layer=0, flags=0, split_pages=0, what=""):
+    run = Run(batch, layer)
+    run.append()
+    run.forward(flags=flags, split_pages=split_pages)
+    code, bits = run.status()
+    assert code == 0, f"device status bits {bits}"
+    ref_out, ref_lse, (okc, ovc) = oracle_full(batch, layer)
+    assert np.array_equal(W.to_host(run.kc), okc), "k pool differs after append"
+    assert np.array_equal(W.to_host(run.vc), ovc), "v pool differs after append"
+    got_out, got_lse = run.out_host()
+    return run, assert_parity(got_out, got_lse, ref_out, ref_lse, what or batch.name)
+
+
+def test_tiny_decode():
+    _full_check(W.config_tiny())
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_fuzz_small_batches(seed):
+    _full_check(W.fuzz_batch(seed), what=f"fuzz{seed}")
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_fuzz_long_rows(seed):
+    # a few rows long enough for many splits and several append tiles
+    _full_check(W.fuzz_batch(1000 + seed, max_len=3000, max_chunk=300), what=f"fuzzlong{seed}")
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_peaked_inputs(seed):
+    rng = np.random.default_rng(200 + seed)
+    B = int(rng.integers(2, 7))
+    S = rng.integers(20, 1500, size=B)
+    L = np.where(rng.random(B) < 0.5, 1, np.minimum(S, rng.integers(2, 200, size=B)))
+    b = W.build_batch("peaked", 300 + seed, S, L, 64, 8, layer_windows=(int(rng.choice([0, 128])),), peaked=True)
+    _full_check(b, what=f"peaked{seed}")
+
+
+@pytest.mark.parametrize("split_pages", [1, 2, 3, 8, 1000])
+def test_split_length_does_not_change_results(split_pages):
+    b = W.build_batch("splits", 55, [700, 33, 2049, 16, 1], [1, 1, 1, 1, 1], 32, 8)
+    run, _ = _full_check(b, split_pages=split_pages, what=f"split{split_pages}")
+    hdr = run.header()
+    if split_pages <= 3:
+        assert hdr["n_merge"] > 0 and hdr["n_decode"] > b.num_seqs
+
+
+@pytest.mark.parametrize("window", [1, 16, 128, 1000])
+def test_sliding_window(window):
+    rng = np.random.default_rng(window)
+    B = 6
+    S = rng.integers(1, 2500, size=B)
+    L = np.where(np.arange(B) % 2 == 0, 1, np.minimum(S, rng.integers(2, 300, size=B)))
+    b = W.build_batch("win", 77 + window, S, L, 64, 8, layer_windows=(window,))
+    _full_check(b, what=f"window{window}")
+
+
+def _grouped_batch(seed, groups=3, group_size=8, append_frac=0.25):
+    rng = np.random.default_rng(seed)
+    grp = np.repeat(np.arange(groups), group_size)
+    prompt = rng.integers(100, 1200, size=groups)[grp]
+    B = groups * group_size
+    L = np.where(rng.random(B) < append_frac, rng.integers(2, 100, size=B), 1)
+    S = prompt + rng.integers(0, 600, size=B) + L
+    shared = prompt // 16
+    return W.build_batch(f"groups{seed}", seed, S, L, 64, 8, shared_prefix_pages=shared, prompt_lens=prompt,
+                         group_of_row=grp)
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_cascade_matches_oracle_and_flat(seed):
+    b = _grouped_batch(seed)
+    run, _ = _full_check(b, what="cascade")
+    hdr = run.header()
+    assert hdr["n_cascade"] > 0, "shared prompt pages were not detected"
+    casc_out, casc_lse = run.out_host()
+    run2, _ = _full_check(b, flags=mcpu.FLAG_NO_CASCADE, what="flat")
+    assert run2.header()["n_cascade"] == 0
+    flat_out, flat_lse = run2.out_host()
+    assert np.max(np.abs(casc_out - flat_out)) <= 2e-2
+    assert np.max(np.abs(casc_lse - flat_lse)) <= 1e-3
+
+
+def test_groups_larger_than_a_cascade_item():
+    # 13 decode members in one group: split into balanced subgroups
+    b = _grouped_batch(9, groups=2, group_size=13, append_frac=0.0)
+    run, _ = _full_check(b, what="biggroup")
+    assert run.header()["n_cascade"] >= 2
+
+
+def test_rows_without_queries_and_single_key_rows():
+    b = W.build_batch("edge", 91, [1, 5, 16, 17, 40], [1, 0, 16, 0, 3], 16, 2)
+    run, _ = _full_check(b, what="edge")
+
+
+@pytest.mark.parametrize("group", [1, 2, 4, 8])
+def test_gqa_ratios(group):
+    b = W.build_batch(f"g{group}", 31 + group, [300, 77, 1200], [1, 50, 1], 2 * group, 2)
+    _full_check(b, what=f"gqa{group}")
+
+
+# ---------------------------------------------------------------- full sizes
+
+
+def _sampled_check(batch, rows, n_per_row, seed, layer=0, run=None):
+    if run is None:
+        run = Run(batch, layer)
+        run.append()
+        run.forward()
+    code, bits = run.status()
+    assert code == 0, f"device status bits {bits}"
+    rng = np.random.default_rng(seed)
+    toks, heads, ref_out, ref_lse = oracle_sampled(batch, rows, n_per_row, rng, layer)
+    got_out, got_lse = run.out_host()
+    return assert_parity(got_out[toks, heads], got_lse[toks, heads], ref_out, ref_lse,
+                         f"{batch.name} layer {layer}")
+
+
+def test_decode_batch_full():
+    b = W.config_decode(device="cuda")
+    run = Run(b)
+    run.append()
+    run.forward()
+    code, _ = run.status()
+    assert code == 0
+    ref_out, ref_lse, _ = oracle_full(b)
+    got_out, got_lse = run.out_host()
+    assert_parity(got_out, got_lse, ref_out, ref_lse, "decode_b64")
+
+
+def test_mixed_batch_sampled():
+    b = W.config_mixed(device="cuda")
+    L = b.q_lens
+    app = list(np.nonzero(L > 1)[0])
+    dec = list(np.nonzero(L == 1)[0])
+    rng = np.random.default_rng(5)
+    rows = sorted(app[:6] + list(rng.choice(dec, size=10, replace=False)))
+    _sampled_check(b, rows, n_per_row=24, seed=6)
+
+
+def test_long_horizon_sampled():
+    b = W.config_long(device="cuda")
+    order = np.argsort(b.seq_lens)
+    rows = sorted(list(order[:3]) + list(order[-4:]) + list(order[len(order) // 2: len(order) // 2 + 3]))
+    _sampled_check(b, rows, n_per_row=16, seed=7)
+
+
+def test_rollout_step_sampled_every_layer():
+    b = W.config_rollout(device="cuda")
+    L = b.q_lens
+    rng = np.random.default_rng(8)
+    app = list(np.nonzero(L > 1)[0])
+    dec = list(np.nonzero(L == 1)[0])
+    # one whole GRPO group (shared prompt) plus a few others
+    grp_rows = list(np.nonzero(b.group_of_row == b.group_of_row[dec[0]])[0])
+    rows = sorted(set(grp_rows + app[:3] + list(rng.choice(dec, size=4, replace=False))))
+    for layer in range(len(b.layers)):
+        run = Run(b, layer)
+        run.append()
+        run.forward()
+        if b.layers[layer].sliding_window == 0:
+            assert run.header()["n_cascade"] > 0
+        _sampled_check(b, rows, n_per_row=6, seed=100 + layer, layer=layer, run=run)
+        del run
+        torch.cuda.empty_cache()
