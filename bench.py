@@ -52,6 +52,7 @@ WORKLOAD_DESC = {
     "decode": "decode batch: 64 rows, S~U[2048,16384], 64q/8kv, D=64, page 16, bf16",
     "mixed": "mixed multi-turn batch: 256 rows, prior~U[4096,32768], 224 decode + 32 append rows "
              "(chunk logU[64,2048]), 64q/8kv, D=64, page 16, bf16",
+    "mixed_small": "mixed batch at 64 rows (8 append), same distributions; profiling case",
     "long": "long-horizon decode: 512 rows, S lognormal(median 12288, sigma 1) in [512,65536], "
             "1/3 in [49152,65536], 64q/8kv, D=64, page 16, bf16",
     "rollout": "rollout step: 24 layers alternating SWA-128/full, 48 GRPO groups x 8 rows sharing prompt "
@@ -235,7 +236,8 @@ class Stepper:
 
 def make_batch(name, dev, rank):
     fn = W.CONFIGS[name]
-    seed = {"tiny": 1001, "decode": 1002, "mixed": 1003, "long": 1004, "rollout": 1005}[name] + 7 * rank
+    seed = {"tiny": 1001, "decode": 1002, "mixed": 1003, "mixed_small": 1013, "long": 1004,
+            "rollout": 1005}[name] + 7 * rank
     return fn(seed=seed, device=dev)
 
 

@@ -50,7 +50,7 @@
  *                 softmax normaliser sum_j exp(scale * q.k_j); -inf if empty)
  *
  * Supported now: D = 64, page_size = 16, H_q / H_kv in {1, 2, 4, 8},
- * num_seqs <= 4096. Anything else returns MCPU_ERR_UNSUPPORTED.
+ * num_seqs <= 2048. Anything else returns MCPU_ERR_UNSUPPORTED.
  */
 #ifndef MCPU_H
 #define MCPU_H
@@ -90,7 +90,8 @@ typedef struct mcpu_dims {
 } mcpu_dims;
 
 /* Optional knobs of the forward pass; pass NULL for the defaults. */
-#define MCPU_FLAG_NO_CASCADE 0x1u   /* never run the shared-prefix (cascade) pass */
+#define MCPU_FLAG_NO_CASCADE 0x1u       /* never run the shared-prefix (cascade) pass */
+#define MCPU_FLAG_MMA_SYNC_APPEND 0x2u  /* append chunks on the mma.sync kernel instead of tcgen05 */
 typedef struct mcpu_options {
   uint32_t flags;             /* MCPU_FLAG_* */
   int32_t split_pages;        /* > 0: KV split length of decode rows, in pages (0 = auto) */

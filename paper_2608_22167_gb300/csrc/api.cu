@@ -19,6 +19,9 @@ cudaError_t prepare_decode_kernels(int* bpsm_decode, int* bpsm_cascade);
 cudaError_t launch_append(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
                           cudaStream_t stream);
 cudaError_t prepare_append_kernel(int* bpsm);
+cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
+                             const AttnParams& p, int grid, cudaStream_t stream);
+cudaError_t prepare_append_tc_kernel(int* bpsm);
 cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
                              const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
@@ -35,7 +38,7 @@ constexpr int kMaxDevices = 64;
 struct DeviceState {
   bool ready = false;
   int sms = 0;
-  int bpsm_decode = 0, bpsm_cascade = 0, bpsm_append = 0;
+  int bpsm_decode = 0, bpsm_cascade = 0, bpsm_append = 0, bpsm_append_tc = 0;
 };
 
 std::mutex g_mu;
@@ -62,7 +65,9 @@ mcpu_status device_state(DeviceState** out) {
     if (prepare_plan_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
     if (prepare_decode_kernels(&st.bpsm_decode, &st.bpsm_cascade) != cudaSuccess) return MCPU_ERR_CUDA;
     if (prepare_append_kernel(&st.bpsm_append) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1) return MCPU_ERR_CUDA;
+    if (prepare_append_tc_kernel(&st.bpsm_append_tc) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1 || st.bpsm_append_tc < 1)
+      return MCPU_ERR_CUDA;
     st.ready = true;
   }
   *out = &st;
@@ -77,6 +82,19 @@ bool encode_pool(CUtensorMap* map, const void* pool, int64_t rows) {
   cuuint32_t box[2] = {(cuuint32_t)kHeadDim, (cuuint32_t)kPage};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(pool), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// 3-D view of q [T, H_q, D]: boxes of (128 / g) tokens x the g heads of one kv
+// head x 64 dims, i.e. one 128-row query tile, 128-byte swizzle.
+bool encode_query(CUtensorMap* map, const void* q, int32_t total_q, int32_t num_q_heads, int32_t group) {
+  cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)num_q_heads, (cuuint64_t)total_q};
+  cuuint64_t strides[2] = {(cuuint64_t)kRowBytes, (cuuint64_t)kRowBytes * num_q_heads};
+  cuuint32_t box[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)group, (cuuint32_t)(128 / group)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -173,8 +191,11 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   if (st != MCPU_OK) return st;
 
   const int64_t rows = (int64_t)dims->num_pages * dims->num_kv_heads * kPage;
-  CUtensorMap kmap, vmap;
+  const bool legacy_append = opts && (opts->flags & MCPU_FLAG_MMA_SYNC_APPEND);
+  const int group = dims->num_q_heads / dims->num_kv_heads;
+  CUtensorMap kmap, vmap, qmap;
   if (!encode_pool(&kmap, k_cache, rows) || !encode_pool(&vmap, v_cache, rows)) return MCPU_ERR_INVALID_ARG;
+  if (!legacy_append && !encode_query(&qmap, q, dims->total_q, dims->num_q_heads, group)) return MCPU_ERR_INVALID_ARG;
 
   AttnParams p;
   p.q = static_cast<const __nv_bfloat16*>(q);
@@ -198,6 +219,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   p.forced_split_pages = opts ? opts->split_pages : 0;
   p.cascade_enabled = (opts && (opts->flags & MCPU_FLAG_NO_CASCADE)) ? 0 : 1;
   p.oob_row = (int32_t)rows;
+  p.append_tile_tok = (legacy_append ? kAppendRowsMin : 128) / p.group;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   void* const* ev = opts ? opts->phase_events : nullptr;
@@ -212,7 +234,12 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   if (e == cudaSuccess) e = mark(2);
   if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s);
   if (e == cudaSuccess) e = mark(3);
-  if (e == cudaSuccess) e = launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
+  if (e == cudaSuccess) {
+    if (legacy_append)
+      e = launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
+    else
+      e = launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
+  }
   if (e == cudaSuccess) e = mark(4);
   if (e == cudaSuccess) {
     const int want = (p.num_seqs * p.num_q_heads + 7) / 8;

@@ -17,14 +17,14 @@ constexpr int kHeadDim = 64;          // D; one key row = 128 bytes of bf16
 constexpr int kPage = 16;             // tokens per page
 constexpr int kRowBytes = kHeadDim * 2;
 constexpr int kTileBytes = kPage * kRowBytes;  // one (page, kv head) block: 2 KiB
-constexpr int kMaxSeqs = 4096;        // rows per call handled by the planner
+constexpr int kMaxSeqs = 2048;        // rows per call handled by the planner
 constexpr int kPlanThreads = 1024;
 constexpr int kRowsPerPlanThread = kMaxSeqs / kPlanThreads;
 constexpr int kMaxGroup = 8;          // largest supported H_q / H_kv
 constexpr int kSplitBudget = 4096;    // bound on member-weighted KV splits per call
 constexpr int kMinSplitPages = 8;     // shortest split of a decode row, in pages
 constexpr int kMinSharedPages = 4;    // shortest prefix worth a cascade pass
-constexpr int kAppendRows = 64;       // query rows (tokens x heads) per append tile
+constexpr int kAppendRowsMin = 64;    // smallest append tile (query rows = tokens x heads)
 
 // Status bits, OR-ed into the first word of the workspace. They are sticky
 // until the caller resets them.
@@ -82,7 +82,7 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 __host__ __device__ inline WorkspaceLayout workspace_layout(int32_t num_seqs, int32_t total_q,
                                                             int32_t num_q_heads, int32_t group) {
   WorkspaceLayout w;
-  int32_t tile_tok = kAppendRows / group;
+  int32_t tile_tok = kAppendRowsMin / group;
   w.max_decode = num_seqs + kSplitBudget + 1;
   w.max_cascade = num_seqs / 2 + kSplitBudget + 1;
   w.max_append = total_q / tile_tok + num_seqs + 1;
@@ -118,6 +118,7 @@ struct AttnParams {
   int32_t forced_split_pages;    // > 0: use this split length
   int32_t cascade_enabled;
   int32_t oob_row;               // y coordinate just past the pool, read as zeros
+  int32_t append_tile_tok;       // tokens per append tile (tile rows / group)
 };
 
 __device__ __forceinline__ PlanHeader* header(const AttnParams& p) {

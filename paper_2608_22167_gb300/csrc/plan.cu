@@ -9,6 +9,10 @@
 // same physical pages (the G samples of a GRPO task sharing their prompt,
 // paper §4), the shared prefix that one cascade pass reads once for the
 // whole group; for append rows, the query tiles of the chunk kernel.
+//
+// Per-row quantities are held in shared memory; every count becomes an
+// offset by a CTA-wide prefix sum, and the records are then written by all
+// threads in parallel (each finds its row by binary search over the offsets).
 #include "common.cuh"
 
 namespace mcpu {
@@ -52,34 +56,71 @@ __device__ int cta_scan(int v, int* total, ScanBuf& sb) {
   return res;
 }
 
-// Exclusive scan of R values per thread (rows tid*R .. tid*R+R-1).
-__device__ void cta_scan_rows(const int (&v)[R], int (&out)[R], int* total, ScanBuf& sb) {
-  int s = 0;
-#pragma unroll
-  for (int i = 0; i < R; ++i) s += v[i];
-  int base = cta_scan(s, total, sb);
+// Exclusive scan of a per-row array in shared memory (rows tid*R .. +R-1),
+// written back in place; returns the total.
+__device__ int scan_rows(int* a, int B, ScanBuf& sb) {
+  int v[R], s = 0;
 #pragma unroll
   for (int i = 0; i < R; ++i) {
-    out[i] = base;
+    const int r = threadIdx.x * R + i;
+    v[i] = r < B ? a[r] : 0;
+    s += v[i];
+  }
+  int total;
+  int base = cta_scan(s, &total, sb);
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    const int r = threadIdx.x * R + i;
+    if (r < B) a[r] = base;
     base += v[i];
   }
+  __syncthreads();
+  return total;
+}
+
+// Last row r with off[r] <= e (rows with no records share the next row's
+// offset, so the last one is always a row that owns record e).
+__device__ __forceinline__ int owner_row(const int* off, int B, int e) {
+  int lo = 0, hi = B;  // off[lo] <= e < off[hi] (off[B] = +inf)
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (off[mid] <= e) lo = mid; else hi = mid;
+  }
+  return lo;
 }
 
 __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
 
 }  // namespace
 
-// Dynamic shared memory: per-row arrays (kMaxSeqs entries each).
+// Row flags
+constexpr int kFlagMember = 1;    // decode row served by a cascade pass
+constexpr int kFlagDirect = 2;    // decode row with one part: writes out/lse itself
+constexpr int kFlagSubFirst = 4;  // first member of its cascade subgroup
+
 struct PlanSmem {
-  int S[kMaxSeqs];
-  int lcp[kMaxSeqs];
-  int gid[kMaxSeqs];
-  int grp_pages[kMaxSeqs];   // shared full pages of a group (min over the run)
-  int grp_ndec[kMaxSeqs];    // decode rows in the group
-  int grp_base[kMaxSeqs];    // smallest member rank in the group
-  signed char kind[kMaxSeqs];  // 0 none / invalid, 1 decode, 2 append
+  int S[kMaxSeqs];          // seq_len, -1 if the row is invalid
+  int L[kMaxSeqs];
+  int Q0[kMaxSeqs];         // first query token
+  int lcp[kMaxSeqs];        // leading pages equal to the previous row's
+  int gid[kMaxSeqs];        // run (group) id
+  int grp_pages[kMaxSeqs];  // per group: shared full pages
+  int grp_ndec[kMaxSeqs];   // per group: decode rows
+  int grp_base[kMaxSeqs];   // per group: smallest member rank
+  int mrank[kMaxSeqs];      // member rank (cascade member array index)
+  int own_pb[kMaxSeqs];     // first page of the row's own decode range
+  int n_cs[kMaxSeqs];       // cascade splits covering the row
+  int part_off[kMaxSeqs];
+  int item_off[kMaxSeqs];   // decode records
+  int sg_off[kMaxSeqs];     // cascade records (subgroup-first rows only)
+  int tile_off[kMaxSeqs];   // append records
+  int sub_first_idx[kMaxSeqs];  // first member index of the row's subgroup
+  int sub_n[kMaxSeqs];          // members in the row's subgroup
+  unsigned char kind[kMaxSeqs];   // 0 none / invalid, 1 decode, 2 append
+  unsigned char flags[kMaxSeqs];
   ScanBuf sb;
   int bad_global;
+  int split_pages;
 };
 
 __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
@@ -88,12 +129,11 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   PlanHeader* hdr = header(p);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int B = p.num_seqs;
-  const int Hkv = p.num_kv_heads;
-  const int tile_tok = kAppendRows / p.group;
-  const int sub_cap = 32 / p.group;  // query vectors of a cascade item: 32
+  const int tile_tok = p.append_tile_tok;
+  const int sub_cap = 32 / p.group;  // rows per cascade item (32 query vectors)
 
   if (tid == 0) {
-    int bad = (p.qsl[0] != 0 || p.qsl[B] != p.total_q) ? 1 : 0;
+    const int bad = (p.qsl[0] != 0 || p.qsl[B] != p.total_q) ? 1 : 0;
     sm.bad_global = bad;
     if (bad) atomicOr(&hdr->status, kStatusBadLengths);
   }
@@ -108,30 +148,20 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   }
 
   // ---- phase 1: per-row kind and lengths
-  int S[R], L[R], Q0[R], kind[R];
-#pragma unroll
-  for (int i = 0; i < R; ++i) {
-    const int r = tid * R + i;
-    S[i] = L[i] = Q0[i] = kind[i] = 0;
-    if (r < B) {
-      const int q0 = p.qsl[r], q1 = p.qsl[r + 1];
-      const int len = q1 - q0, s = p.seq_lens[r];
-      const bool bad = len < 0 || s < len || s > p.max_pages * kPage;
-      if (bad) {
-        atomicOr(&hdr->status, kStatusBadLengths);
-      } else {
-        S[i] = s;
-        L[i] = len;
-        Q0[i] = q0;
-        kind[i] = len == 0 ? 0 : (len == 1 ? 1 : 2);
-      }
-      sm.S[r] = bad ? -1 : s;
-      sm.kind[r] = (signed char)kind[i];
-      sm.lcp[r] = 0;
-      sm.grp_pages[r] = 0x7fffffff;
-      sm.grp_ndec[r] = 0;
-      sm.grp_base[r] = 0x7fffffff;
-    }
+  for (int r = tid; r < B; r += kPlanThreads) {
+    const int q0 = p.qsl[r], q1 = p.qsl[r + 1];
+    const int len = q1 - q0, s = p.seq_lens[r];
+    const bool bad = len < 0 || s < len || s > p.max_pages * kPage;
+    if (bad) atomicOr(&hdr->status, kStatusBadLengths);
+    sm.S[r] = bad ? -1 : s;
+    sm.L[r] = bad ? 0 : len;
+    sm.Q0[r] = q0;
+    sm.kind[r] = bad ? 0 : (len == 0 ? 0 : (len == 1 ? 1 : 2));
+    sm.lcp[r] = 0;
+    sm.grp_pages[r] = 0x7fffffff;
+    sm.grp_ndec[r] = 0;
+    sm.grp_base[r] = 0x7fffffff;
+    sm.flags[r] = 0;
   }
   __syncthreads();
 
@@ -160,82 +190,88 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     }
   }
   __syncthreads();
-
   // group id = (number of run starts up to and including r) - 1
+  for (int r = tid; r < B; r += kPlanThreads)
+    sm.gid[r] = (r == 0 || !cascade || sm.lcp[r] < kMinSharedPages) ? 1 : 0;
+  __syncthreads();
   {
-    int st[R], ex[R], tot;
+    int st[R];
 #pragma unroll
     for (int i = 0; i < R; ++i) {
       const int r = tid * R + i;
-      st[i] = (r < B && (r == 0 || !cascade || sm.lcp[r] < kMinSharedPages)) ? 1 : 0;
+      st[i] = r < B ? sm.gid[r] : 0;
     }
-    cta_scan_rows(st, ex, &tot, sm.sb);
+    __syncthreads();
+    int total, sum = 0;
+#pragma unroll
+    for (int i = 0; i < R; ++i) sum += st[i];
+    int base = cta_scan(sum, &total, sm.sb);
 #pragma unroll
     for (int i = 0; i < R; ++i) {
       const int r = tid * R + i;
-      if (r < B) sm.gid[r] = ex[i] + st[i] - 1;
+      base += st[i];
+      if (r < B) sm.gid[r] = base - 1;
     }
   }
   __syncthreads();
   if (cascade) {
-#pragma unroll
-    for (int i = 0; i < R; ++i) {
-      const int r = tid * R + i;
-      if (r >= B) continue;
+    for (int r = tid; r < B; r += kPlanThreads) {
       const int g = sm.gid[r];
       if (r > 0 && sm.gid[r - 1] == g) atomicMin(&sm.grp_pages[g], sm.lcp[r]);
-      if (kind[i] == 1) {
-        atomicMin(&sm.grp_pages[g], S[i] / kPage);
+      if (sm.kind[r] == 1) {
+        atomicMin(&sm.grp_pages[g], sm.S[r] / kPage);
         atomicAdd(&sm.grp_ndec[g], 1);
       }
     }
   }
   __syncthreads();
-
   // members: decode rows of a group with >= 2 decode rows and a long enough prefix
-  int member[R], mrank[R], n_members_total;
-  {
-#pragma unroll
-    for (int i = 0; i < R; ++i) {
-      const int r = tid * R + i;
-      member[i] = 0;
-      if (cascade && r < B && kind[i] == 1) {
-        const int g = sm.gid[r];
-        member[i] = (sm.grp_ndec[g] >= 2 && sm.grp_pages[g] >= kMinSharedPages) ? 1 : 0;
-      }
+  for (int r = tid; r < B; r += kPlanThreads) {
+    int m = 0;
+    if (cascade && sm.kind[r] == 1) {
+      const int g = sm.gid[r];
+      m = (sm.grp_ndec[g] >= 2 && sm.grp_pages[g] >= kMinSharedPages) ? 1 : 0;
     }
-    cta_scan_rows(member, mrank, &n_members_total, sm.sb);
-#pragma unroll
-    for (int i = 0; i < R; ++i)
-      if (member[i]) atomicMin(&sm.grp_base[sm.gid[tid * R + i]], mrank[i]);
+    sm.mrank[r] = m;
+    if (m) sm.flags[r] |= kFlagMember;
   }
+  __syncthreads();
+  scan_rows(sm.mrank, B, sm.sb);
+  for (int r = tid; r < B; r += kPlanThreads)
+    if (sm.flags[r] & kFlagMember) atomicMin(&sm.grp_base[sm.gid[r]], sm.mrank[r]);
   __syncthreads();
 
   // ---- phase 3: split length
-  int own_pb[R], own_pe[R], gpages[R], nsub[R], sub_idx[R], sub_first[R];
   int w_m = 0, w_lb = 0;
-#pragma unroll
-  for (int i = 0; i < R; ++i) {
-    const int r = tid * R + i;
-    own_pb[i] = own_pe[i] = gpages[i] = nsub[i] = sub_idx[i] = sub_first[i] = 0;
-    if (r >= B || kind[i] != 1) continue;
-    const int first_key = p.window > 0 ? max(0, S[i] - p.window) : 0;
-    own_pe[i] = cdiv(S[i], kPage);
-    own_pb[i] = first_key / kPage;
-    if (member[i]) {
+  for (int r = tid; r < B; r += kPlanThreads) {
+    sm.own_pb[r] = 0;
+    sm.n_cs[r] = 0;
+    sm.sub_first_idx[r] = 0;
+    sm.sub_n[r] = 0;
+    if (sm.kind[r] != 1) continue;
+    const int S = sm.S[r];
+    const int first_key = p.window > 0 ? max(0, S - p.window) : 0;
+    const int pe = cdiv(S, kPage);
+    int pb = first_key / kPage;
+    int gp = 0;
+    if (sm.flags[r] & kFlagMember) {
       const int g = sm.gid[r];
       const int nd = sm.grp_ndec[g];
-      gpages[i] = sm.grp_pages[g];
-      own_pb[i] = gpages[i];
-      nsub[i] = cdiv(nd, sub_cap);
-      const int idx = mrank[i] - sm.grp_base[g];
-      sub_idx[i] = idx * nsub[i] / nd;
-      // first member index of this subgroup: ceil(sub * nd / nsub)
-      sub_first[i] = (idx == cdiv(sub_idx[i] * nd, nsub[i])) ? 1 : 0;
+      gp = sm.grp_pages[g];
+      pb = gp;
+      const int nsub = cdiv(nd, sub_cap);
+      const int idx = sm.mrank[r] - sm.grp_base[g];
+      const int sub = idx * nsub / nd;
+      const int first = cdiv(sub * nd, nsub), next = cdiv((sub + 1) * nd, nsub);
+      sm.sub_first_idx[r] = sm.grp_base[g] + first;
+      sm.sub_n[r] = next - first;
+      if (idx == first) sm.flags[r] |= kFlagSubFirst;
     }
-    const int own = own_pe[i] - own_pb[i];
-    w_m += own + (member[i] ? gpages[i] : 0);
-    w_lb += own + (sub_first[i] ? gpages[i] : 0);
+    sm.own_pb[r] = pb;
+    sm.n_cs[r] = gp;  // shared pages for now; split count after C is known
+    const int own = pe - pb;
+    w_m += own + gp;
+    w_lb += own + ((sm.flags[r] & kFlagSubFirst) ? gp : 0);
   }
   int tot_wm, tot_wlb;
   cta_scan(w_m, &tot_wm, sm.sb);
@@ -246,41 +282,36 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     C = max(p.forced_split_pages, c_bound);
   } else {
     const long long denom = 4LL * max(p.total_warps_hint, 1);
-    const int c_lb = (int)((((long long)tot_wlb) * Hkv + denom - 1) / denom);
+    const int c_lb = (int)((((long long)tot_wlb) * p.num_kv_heads + denom - 1) / denom);
     C = max(kMinSplitPages, max(c_lb, c_bound));
   }
 
-  // ---- phase 4: decode items, partial slots, merge rows
-  int n_own[R], n_cs[R], parts[R], direct[R];
-#pragma unroll
-  for (int i = 0; i < R; ++i) {
-    n_own[i] = (kind[i] == 1) ? cdiv(own_pe[i] - own_pb[i], C) : 0;
-    n_cs[i] = member[i] ? cdiv(gpages[i], C) : 0;
-    parts[i] = n_own[i] + n_cs[i];
-    direct[i] = (kind[i] == 1 && !member[i] && parts[i] == 1) ? 1 : 0;
+  // ---- phase 4: per-row counts -> offsets
+  for (int r = tid; r < B; r += kPlanThreads) {
+    int n_own = 0, n_cs = 0, parts = 0, tiles = 0, sg = 0, direct = 0;
+    if (sm.kind[r] == 1) {
+      const int pe = cdiv(sm.S[r], kPage);
+      n_own = cdiv(pe - sm.own_pb[r], C);
+      const bool member = sm.flags[r] & kFlagMember;
+      n_cs = member ? cdiv(sm.n_cs[r], C) : 0;
+      parts = n_own + n_cs;
+      direct = (!member && parts == 1) ? 1 : 0;
+      if (direct) sm.flags[r] |= kFlagDirect;
+      if (sm.flags[r] & kFlagSubFirst) sg = n_cs;
+    } else if (sm.kind[r] == 2) {
+      tiles = cdiv(sm.L[r], tile_tok);
+    }
+    sm.n_cs[r] = n_cs;
+    sm.part_off[r] = direct ? 0 : parts;
+    sm.item_off[r] = n_own;
+    sm.sg_off[r] = sg;
+    sm.tile_off[r] = tiles;
   }
-  int pc[R], part_off[R], item_off[R], is_merge[R], merge_off[R];
-  int tot_parts, tot_items, tot_merge;
-#pragma unroll
-  for (int i = 0; i < R; ++i) {
-    pc[i] = (kind[i] == 1 && !direct[i]) ? parts[i] : 0;
-    is_merge[i] = pc[i] > 0 ? 1 : 0;
-  }
-  cta_scan_rows(pc, part_off, &tot_parts, sm.sb);
-  cta_scan_rows(n_own, item_off, &tot_items, sm.sb);
-  cta_scan_rows(is_merge, merge_off, &tot_merge, sm.sb);
-
-  // ---- phase 5: cascade subgroups (one record per split of each subgroup)
-  int sg_splits[R], sg_off[R], tot_cascade;
-#pragma unroll
-  for (int i = 0; i < R; ++i) sg_splits[i] = sub_first[i] ? n_cs[i] : 0;
-  cta_scan_rows(sg_splits, sg_off, &tot_cascade, sm.sb);
-
-  // ---- phase 6: append tiles
-  int tiles[R], tile_off[R], tot_tiles;
-#pragma unroll
-  for (int i = 0; i < R; ++i) tiles[i] = kind[i] == 2 ? cdiv(L[i], tile_tok) : 0;
-  cta_scan_rows(tiles, tile_off, &tot_tiles, sm.sb);
+  __syncthreads();
+  const int tot_parts = scan_rows(sm.part_off, B, sm.sb);
+  const int tot_items = scan_rows(sm.item_off, B, sm.sb);
+  const int tot_cascade = scan_rows(sm.sg_off, B, sm.sb);
+  const int tot_tiles = scan_rows(sm.tile_off, B, sm.sb);
 
   const bool overflow = tot_items > p.lay.max_decode || tot_cascade > p.lay.max_cascade ||
                         tot_tiles > p.lay.max_append || tot_parts > p.lay.max_parts;
@@ -300,84 +331,92 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   AppendItem* aitems = reinterpret_cast<AppendItem*>(p.ws + p.lay.append_items);
   MergeRow* mrows = reinterpret_cast<MergeRow*>(p.ws + p.lay.merge_rows);
 
-#pragma unroll
-  for (int i = 0; i < R; ++i) {
-    const int r = tid * R + i;
-    if (r >= B) continue;
-    if (kind[i] == 1) {
-      const int first_key = p.window > 0 ? max(0, S[i] - p.window) : 0;
-      for (int k = 0; k < n_own[i]; ++k) {
-        DecodeItem it;
-        it.row = r;
-        it.token = Q0[i];
-        it.seq_len = S[i];
-        it.first_key = first_key;
-        it.page_begin = own_pb[i] + k * C;
-        it.page_end = min(own_pe[i], own_pb[i] + (k + 1) * C);
-        it.slot = direct[i] ? -1 : part_off[i] + n_cs[i] + k;
-        it.pad = 0;
-        ditems[item_off[i] + k] = it;
-      }
-      if (is_merge[i]) {
-        MergeRow m;
-        m.token = Q0[i];
-        m.n_parts = parts[i];
-        m.part_off = part_off[i];
-        m.pad = 0;
-        mrows[merge_off[i]] = m;
-      }
-      if (member[i]) {
-        CascadeMember cm;
-        cm.row = r;
-        cm.token = Q0[i];
-        cm.part_off = part_off[i];
-        cm.pad = 0;
-        members[mrank[i]] = cm;
-      }
-      if (sub_first[i]) {
-        const int g = sm.gid[r];
-        const int nd = sm.grp_ndec[g];
-        const int first = cdiv(sub_idx[i] * nd, nsub[i]);
-        const int next = cdiv((sub_idx[i] + 1) * nd, nsub[i]);
-        for (int k = 0; k < n_cs[i]; ++k) {
-          CascadeItem c;
-          c.member_off = sm.grp_base[g] + first;
-          c.n_members = next - first;
-          c.page_begin = k * C;
-          c.page_end = min(gpages[i], (k + 1) * C);
-          c.split = k;
-          c.first_row = r;
-          c.pad0 = c.pad1 = 0;
-          citems[sg_off[i] + k] = c;
-        }
-      }
-    } else if (kind[i] == 2) {
-      for (int k = 0; k < tiles[i]; ++k) {
-        AppendItem a;
-        a.row = r;
-        a.token_begin = Q0[i] + k * tile_tok;
-        a.n_tok = min(tile_tok, L[i] - k * tile_tok);
-        a.seq_len = S[i];
-        a.pos_begin = S[i] - L[i] + k * tile_tok;
-        a.key_begin = p.window > 0 ? max(0, a.pos_begin - p.window + 1) : 0;
-        a.key_end = a.pos_begin + a.n_tok;
-        a.pad = 0;
-        aitems[tile_off[i] + k] = a;
-      }
+  // ---- phase 5: per-row records (merge rows, cascade members)
+  int is_merge_cnt = 0;
+  {
+    // merge rows get consecutive indices: reuse lcp[] as the scan buffer
+    for (int r = tid; r < B; r += kPlanThreads)
+      sm.lcp[r] = (sm.kind[r] == 1 && !(sm.flags[r] & kFlagDirect)) ? 1 : 0;
+    __syncthreads();
+    is_merge_cnt = scan_rows(sm.lcp, B, sm.sb);
+  }
+  for (int r = tid; r < B; r += kPlanThreads) {
+    if (sm.kind[r] != 1) continue;
+    const int parts = (r + 1 < B ? sm.part_off[r + 1] : tot_parts) - sm.part_off[r];
+    if (!(sm.flags[r] & kFlagDirect)) {
+      MergeRow m;
+      m.token = sm.Q0[r];
+      m.n_parts = parts;
+      m.part_off = sm.part_off[r];
+      m.pad = 0;
+      mrows[sm.lcp[r]] = m;
     }
+    if (sm.flags[r] & kFlagMember) {
+      CascadeMember cm;
+      cm.row = r;
+      cm.token = sm.Q0[r];
+      cm.part_off = sm.part_off[r];
+      cm.pad = 0;
+      members[sm.mrank[r]] = cm;
+    }
+  }
+
+  // ---- phase 6: split records, all threads in parallel
+  for (int e = tid; e < tot_items; e += kPlanThreads) {
+    const int r = owner_row(sm.item_off, B, e);
+    const int k = e - sm.item_off[r];
+    const int S = sm.S[r];
+    const int pe = cdiv(S, kPage);
+    DecodeItem it;
+    it.row = r;
+    it.token = sm.Q0[r];
+    it.seq_len = S;
+    it.first_key = p.window > 0 ? max(0, S - p.window) : 0;
+    it.page_begin = sm.own_pb[r] + k * C;
+    it.page_end = min(pe, sm.own_pb[r] + (k + 1) * C);
+    it.slot = (sm.flags[r] & kFlagDirect) ? -1 : sm.part_off[r] + sm.n_cs[r] + k;
+    it.pad = 0;
+    ditems[e] = it;
+  }
+  for (int e = tid; e < tot_cascade; e += kPlanThreads) {
+    const int r = owner_row(sm.sg_off, B, e);
+    const int k = e - sm.sg_off[r];
+    const int gp = sm.grp_pages[sm.gid[r]];
+    CascadeItem c;
+    c.member_off = sm.sub_first_idx[r];
+    c.n_members = sm.sub_n[r];
+    c.page_begin = k * C;
+    c.page_end = min(gp, (k + 1) * C);
+    c.split = k;
+    c.first_row = r;
+    c.pad0 = c.pad1 = 0;
+    citems[e] = c;
+  }
+  for (int e = tid; e < tot_tiles; e += kPlanThreads) {
+    const int r = owner_row(sm.tile_off, B, e);
+    const int k = e - sm.tile_off[r];
+    const int S = sm.S[r], L = sm.L[r];
+    AppendItem a;
+    a.row = r;
+    a.token_begin = sm.Q0[r] + k * tile_tok;
+    a.n_tok = min(tile_tok, L - k * tile_tok);
+    a.seq_len = S;
+    a.pos_begin = S - L + k * tile_tok;
+    a.key_begin = p.window > 0 ? max(0, a.pos_begin - p.window + 1) : 0;
+    a.key_end = a.pos_begin + a.n_tok;
+    a.pad = 0;
+    aitems[e] = a;
   }
   if (tid == 0) {
     hdr->n_decode = tot_items;
     hdr->n_cascade = tot_cascade;
     hdr->n_append = tot_tiles;
-    hdr->n_merge = tot_merge;
+    hdr->n_merge = is_merge_cnt;
     hdr->split_pages = C;
     hdr->n_parts = tot_parts;
     hdr->append_ticket = 0;
   }
 }
-
-size_t plan_smem_bytes() { return sizeof(PlanSmem); }
 
 cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream) {
   static_assert(sizeof(PlanSmem) < 200 * 1024, "planner shared memory");

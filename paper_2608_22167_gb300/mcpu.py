@@ -35,6 +35,7 @@ STATUS = {
     8: "MCPU_ERR_INTERNAL",
 }
 FLAG_NO_CASCADE = 0x1
+FLAG_MMA_SYNC_APPEND = 0x2
 
 # Device status bits (first word of the workspace).
 STATUS_BAD_PAGE = 1

@@ -52,6 +52,24 @@ def test_peaked_inputs(seed):
     _full_check(b, what=f"peaked{seed}")
 
 
+@pytest.mark.parametrize("seed", range(6))
+def test_append_kernels_agree(seed):
+    # the tcgen05 append kernel (default) and the mma.sync one, both vs the oracle
+    rng = np.random.default_rng(400 + seed)
+    B = int(rng.integers(1, 6))
+    S = rng.integers(2, 3000, size=B)
+    L = np.minimum(S, rng.integers(2, 400, size=B))
+    g = int(rng.choice([1, 2, 4, 8]))
+    W_ = int(rng.choice([0, 0, 128, 37]))
+    b = W.build_batch("appends", 600 + seed, S, L, 2 * g, 2, layer_windows=(W_,))
+    run, _ = _full_check(b, what="tcgen05 append")
+    tc_out, tc_lse = run.out_host()
+    run2, _ = _full_check(b, flags=mcpu.FLAG_MMA_SYNC_APPEND, what="mma.sync append")
+    ms_out, ms_lse = run2.out_host()
+    assert np.max(np.abs(tc_out - ms_out)) <= 2e-2
+    assert np.max(np.abs(tc_lse - ms_lse)) <= 1e-3
+
+
 @pytest.mark.parametrize("split_pages", [1, 2, 3, 8, 1000])
 def test_split_length_does_not_change_results(split_pages):
     b = W.build_batch("splits", 55, [700, 33, 2049, 16, 1], [1, 1, 1, 1, 1], 32, 8)

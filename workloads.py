@@ -328,10 +328,23 @@ def config_rollout(seed=1005, device="cpu", layers=24, window=128, groups=48) ->
     return b
 
 
+def config_mixed_small(seed=1013, device="cpu") -> Batch:
+    """The mixed batch's distributions at a quarter of its rows (64 rows, 8
+    appending): a profiling case whose pool (~2 GB) is still far above L2."""
+    rng = np.random.Generator(np.random.PCG64(seed + 7919))
+    B = 64
+    prior = rng.integers(4096, 32768, size=B, endpoint=True)
+    append_rows = rng.permutation(B)[:8]
+    L = np.ones(B, np.int64)
+    L[append_rows] = _log_uniform_int(rng, 64, 2048, 8)
+    return build_batch("mixed_b64", seed, prior + L, L, 64, 8, device=device)
+
+
 CONFIGS = {
     "tiny": config_tiny,
     "decode": config_decode,
     "mixed": config_mixed,
+    "mixed_small": config_mixed_small,
     "long": config_long,
     "rollout": config_rollout,
 }
