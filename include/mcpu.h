@@ -128,7 +128,7 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
  * Paged attention forward over a mixed batch of decode rows (L_r = 1) and
  * append rows (L_r > 1, causal within the chunk), with an optional sliding
  * window (W <= 0: full context). Rows with L_r = 0 produce nothing.
- * softmax_scale multiplies q.k (1/sqrt(D) for gpt-oss). Rows that are
+ * softmax_scale (> 0, finite) multiplies q.k (1/sqrt(D) for gpt-oss). Rows that are
  * adjacent in the batch and whose block tables start with the same physical
  * pages (a GRPO group's shared prompt) are detected on the device and their
  * common full pages are read once for the whole group (full-context calls

@@ -172,8 +172,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
                                          size_t workspace_bytes, const mcpu_options* opts, mcpu_stream_t stream) {
   mcpu_status st = check_dims(dims);
   if (st != MCPU_OK) return st;
-  if (!(softmax_scale == softmax_scale) || softmax_scale > 3.0e38f || softmax_scale < -3.0e38f)
-    return MCPU_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.f) || softmax_scale > 3.0e38f) return MCPU_ERR_INVALID_ARG;
   if (!workspace) return MCPU_ERR_INVALID_ARG;
   if (workspace_bytes < mcpu_workspace_size(dims)) return MCPU_ERR_WORKSPACE_TOO_SMALL;
   if (!aligned(workspace, 256)) return MCPU_ERR_INVALID_ARG;

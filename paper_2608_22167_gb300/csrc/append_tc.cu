@@ -22,7 +22,9 @@
 //   kv_full/kv_empty   TMA ring; a stage is released by the commit after PV_b
 //   s_full[2]          S_b complete (commit after the 4 QK^T MMAs)
 //   p_full[2]          P_b stored and O rescaled (4 softmax warps arrive)
-//   o_ready            PV_b complete (one phase per key block)
+//   o_ready[2]         PV_b complete, on barrier b & 1 (one phase per two blocks:
+//                      a waiter is never two phases behind, even across the
+//                      item boundary where PV_{b-1} is issued before S_{b+1})
 //   q_full/q_empty     query tile loaded / last QK^T of the item done
 //   o_free             epilogue has read O (next item may overwrite it)
 //   item_full/empty[2] two-slot queue of work items from the producer
@@ -42,7 +44,8 @@ constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
 constexpr float kRescaleThreshold = 8.f;  // log2 units: P may reach 2^8 before O is rescaled
 
 struct TcSmem {  // barriers and small state, after the tiles
-  uint64_t q_full, q_empty, o_ready, o_free;
+  uint64_t q_full, q_empty, o_free;
+  uint64_t o_ready[2];
   uint64_t kv_full[kTcStages], kv_empty[kTcStages];
   uint64_t s_full[2], p_full[2];
   uint64_t item_full[2], item_empty[2];
@@ -88,7 +91,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(bar(st.q_full), 1);
     mbar_init(bar(st.q_empty), 1);
-    mbar_init(bar(st.o_ready), 1);
     mbar_init(bar(st.o_free), 4);
     for (int s = 0; s < kTcStages; ++s) {
       mbar_init(bar(st.kv_full[s]), 1);
@@ -96,6 +98,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar(st.s_full[i]), 1);
+      mbar_init(bar(st.o_ready[i]), 1);
       mbar_init(bar(st.p_full[i]), 4);
       mbar_init(bar(st.item_full[i]), 1);
       mbar_init(bar(st.item_empty[i]), 5);
@@ -119,56 +122,86 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (warp == 4) {
     // ------------------------------------------------------------ producer
+    // The whole warp runs this loop: lane i keeps the page id of page
+    // (chunk + i) for the current and the next 32-page chunk, so the block
+    // table is read ahead with coalesced loads; lane 0 issues the copies.
     if (lane == 0) {
       prefetch_tensormap(&kmap);
       prefetch_tensormap(&vmap);
       prefetch_tensormap(&qmap);
-      const uint64_t pol = policy_evict_first();
-      uint32_t kv_it = 0;
-      for (int i = 0;; ++i) {
-        const int slot = i & 1;
-        if (i >= 2 && !wait_bar(bar(st.item_empty[slot]), ((i >> 1) - 1) & 1, abort_flag)) break;
-        const int idx = atomicAdd(&hdr->append_ticket, 1);
+    }
+    const uint64_t pol = policy_evict_last();
+    uint32_t kv_it = 0;
+    for (int i = 0;; ++i) {
+      const int slot = i & 1;
+      if (i >= 2 && !__all_sync(0xffffffffu, wait_bar(bar(st.item_empty[slot]), ((i >> 1) - 1) & 1, abort_flag)))
+        break;
+      int idx = 0;
+      if (lane == 0) idx = atomicAdd(&hdr->append_ticket, 1);
+      idx = __shfl_sync(0xffffffffu, idx, 0);
+      AppendItem a;
+      if (idx < n_items) a = items[idx / Hkv];
+      if (lane == 0) {
         st.item_idx[slot] = idx;
-        AppendItem a;
-        if (idx < n_items) a = items[idx / Hkv];
         st.items[slot] = a;
         mbar_arrive(bar(st.item_full[slot]));
-        if (idx >= n_items) break;
-        const int kvh = idx % Hkv;
-        if (i >= 1 && !wait_bar(bar(st.q_empty), (i - 1) & 1, abort_flag)) break;
-        mbar_arrive_expect_tx(bar(st.q_full), kTcQBytes);
-        tma_load_3d(sQ, &qmap, 0, kvh * g, a.token_begin, bar(st.q_full));
-        const int* bt_row = p.block_table + (size_t)a.row * p.max_pages;
-        const int kb0 = (a.key_begin / kPage) * kPage;
-        const int nb = (a.key_end - kb0 + kTcKeys - 1) / kTcKeys;
-        const int page_end = (a.key_end + kPage - 1) / kPage;
-        bool ok = true;
-        for (int b = 0; b < nb && ok; ++b, ++kv_it) {
-          const int s = kv_it % kTcStages;
-          if (kv_it >= kTcStages && !wait_bar(bar(st.kv_empty[s]), ((kv_it / kTcStages) - 1) & 1, abort_flag)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(bar(st.kv_full[s]), kTcStageBytes);
-          const uint32_t dk = sKV + s * kTcStageBytes, dv = dk + kTcKvBytes;
-#pragma unroll
-          for (int j = 0; j < kTcKeys / kPage; ++j) {
-            const int lp = kb0 / kPage + b * (kTcKeys / kPage) + j;
-            int y = p.oob_row;
-            if (lp < page_end) {
-              const int pid = __ldg(bt_row + lp);
-              if (pid < 0 || pid >= p.num_pages)
-                raise_status(p, kStatusBadPage);
-              else
-                y = (pid * Hkv + kvh) * kPage;
-            }
-            tma_load_2d(dk + j * kTileBytes, &kmap, 0, y, bar(st.kv_full[s]), pol);
-            tma_load_2d(dv + j * kTileBytes, &vmap, 0, y, bar(st.kv_full[s]), pol);
+      }
+      if (idx >= n_items) break;
+      const int kvh = idx % Hkv;
+      const int* bt_row = p.block_table + (size_t)a.row * p.max_pages;
+      const int pg0 = a.key_begin / kPage;
+      const int kb0 = pg0 * kPage;
+      const int nb = (a.key_end - kb0 + kTcKeys - 1) / kTcKeys;
+      const int page_end = (a.key_end + kPage - 1) / kPage;
+      auto load_chunk = [&](int c) -> int {  // page id of page pg0 + 32c + lane, or -1
+        const int lp = pg0 + 32 * c + lane;
+        int v = -1;
+        if (lp < page_end) {
+          v = __ldg(bt_row + lp);
+          if (v < 0 || v >= p.num_pages) {
+            raise_status(p, kStatusBadPage);
+            v = -1;
           }
         }
-        if (!ok) break;
+        return v;
+      };
+      int pid_cur = load_chunk(0), pid_next = load_chunk(1);
+      if (i >= 1 && !__all_sync(0xffffffffu, wait_bar(bar(st.q_empty), (i - 1) & 1, abort_flag))) break;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(bar(st.q_full), kTcQBytes);
+        tma_load_3d(sQ, &qmap, 0, kvh * g, a.token_begin, bar(st.q_full));
       }
+      bool ok = true;
+      constexpr int kPagesPerBlock = kTcKeys / kPage;  // 8: four blocks per 32-page chunk
+      for (int b = 0; b < nb; ++b, ++kv_it) {
+        if (b > 0 && (b * kPagesPerBlock) % 32 == 0) {
+          pid_cur = pid_next;
+          pid_next = load_chunk(b * kPagesPerBlock / 32 + 1);
+        }
+        const int s = kv_it % kTcStages;
+        if (kv_it >= kTcStages &&
+            !__all_sync(0xffffffffu, wait_bar(bar(st.kv_empty[s]), ((kv_it / kTcStages) - 1) & 1, abort_flag))) {
+          ok = false;
+          break;
+        }
+        const uint32_t dk = sKV + s * kTcStageBytes, dv = dk + kTcKvBytes;
+        const int lane0 = (b * kPagesPerBlock) % 32;
+        int y[kPagesPerBlock];
+#pragma unroll
+        for (int j = 0; j < kPagesPerBlock; ++j) {
+          const int pid = __shfl_sync(0xffffffffu, pid_cur, lane0 + j);
+          y[j] = pid < 0 ? p.oob_row : (pid * Hkv + kvh) * kPage;
+        }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(bar(st.kv_full[s]), kTcStageBytes);
+#pragma unroll
+          for (int j = 0; j < kPagesPerBlock; ++j) {
+            tma_load_2d(dk + j * kTileBytes, &kmap, 0, y[j], bar(st.kv_full[s]), pol);
+            tma_load_2d(dv + j * kTileBytes, &vmap, 0, y[j], bar(st.kv_full[s]), pol);
+          }
+        }
+      }
+      if (!ok) break;
     }
   } else if (warp == 5) {
     // ----------------------------------------------------------- MMA issuer
@@ -201,7 +234,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             tc_mma_ts(tmem + kColO, tmem + (buf ? kColS1 : kColS0) + kk * 8, vdesc, idO, (b > 0 || kk > 0) ? 1u : 0u);
           }
           tc_commit(bar(st.kv_empty[s]));
-          tc_commit(bar(st.o_ready));
+          tc_commit(bar(st.o_ready[gblk & 1]));
           return true;
         };
         for (int b = 0; b < nb; ++b, ++kv_it, ++blk) {
@@ -212,7 +245,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             break;
           }
           // S buffer `buf` was last read by PV_{blk-2}: wait for it
-          if (blk >= 2 && !wait_bar(bar(st.o_ready), (blk - 2) & 1, abort_flag)) {
+          if (blk >= 2 && !wait_bar(bar(st.o_ready[blk & 1]), ((blk - 2) >> 1) & 1, abort_flag)) {
             ok = false;
             break;
           }
@@ -272,45 +305,54 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         tmem_ld_wait();
         const int kbase = kb0 + b * kTcKeys;
         const bool need_mask = (kbase + kTcKeys - 1 > wp_min) || (p.window > 0 && kbase < wp_max - p.window + 1);
-        float mx = -INFINITY;
+        if (need_mask) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+          for (int c = 0; c < 4; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            float x = __uint_as_float(sv[c][e]) * p.scale_log2;
-            if (need_mask) {
+            for (int e = 0; e < 32; ++e) {
               const int j = kbase + 32 * c + e;
-              if (j > pos || j < lo) x = -INFINITY;
+              if (j > pos || j < lo) sv[c][e] = 0xff800000u;  // -inf
             }
-            sv[c][e] = __float_as_uint(x);
-            mx = fmaxf(mx, x);
-          }
         }
+        // row max of the raw scores (the scale is positive), two chains
+        float mxa = -INFINITY, mxb = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            mxa = fmaxf(mxa, __uint_as_float(sv[c][e]));
+            mxb = fmaxf(mxb, __uint_as_float(sv[c][e + 1]));
+          }
+        const float mx = fmaxf(mxa, mxb) * p.scale_log2;
         float alpha = 1.f;
         if (mx > m_ref + kRescaleThreshold) {  // also true for the first finite max
-          alpha = fast_exp2(m_ref - mx);       // 0 when m_ref == -inf
+          alpha = ex2_approx(m_ref - mx);      // 0 when m_ref == -inf
           m_ref = mx;
         }
-        const float mu = m_ref == -INFINITY ? 0.f : m_ref;
-        l *= alpha;
+        const float neg_mu = m_ref == -INFINITY ? 0.f : -m_ref;
+        const float sl2 = p.scale_log2;
+        float la = 0.f, lb = 0.f;
         uint32_t pk[2][32];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            const float p0 = fast_exp2(__uint_as_float(sv[c][e]) - mu);
-            const float p1 = fast_exp2(__uint_as_float(sv[c][e + 1]) - mu);
-            l += p0 + p1;
+            const float p0 = ex2_approx(fmaf(__uint_as_float(sv[c][e]), sl2, neg_mu));
+            const float p1 = ex2_approx(fmaf(__uint_as_float(sv[c][e + 1]), sl2, neg_mu));
+            la += p0;
+            lb += p1;
             pk[c >> 1][(c & 1) * 16 + e / 2] = pack_bf16x2(p0, p1);
           }
         }
-        // PV_{blk-1} must be complete before O is touched or P_blk published
-        if (blk >= 1) {
-          ok = __all_sync(0xffffffffu, wait_bar(bar(st.o_ready), (blk - 1) & 1, abort_flag));
+        l = l * alpha + (la + lb);
+        // O may only be rescaled once PV_{blk-1} has completed. Without a
+        // rescale P_blk is published right away: PV_blk queues behind
+        // PV_{blk-1} on the tensor pipe.
+        if (b > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
+          ok = __all_sync(0xffffffffu,
+                          wait_bar(bar(st.o_ready[(blk - 1) & 1]), ((blk - 1) >> 1) & 1, abort_flag));
           if (!ok) break;
           tc_fence_after();
-        }
-        if (b > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
           uint32_t ov[2][32];
           tmem_ld32(tmem + lane_off + kColO, ov[0]);
           tmem_ld32(tmem + lane_off + kColO + 32, ov[1]);
@@ -332,7 +374,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (!ok) break;
       // epilogue: the last PV of the item
       if (nb > 0) {
-        ok = __all_sync(0xffffffffu, wait_bar(bar(st.o_ready), (blk - 1) & 1, abort_flag));
+        ok = __all_sync(0xffffffffu,
+                        wait_bar(bar(st.o_ready[(blk - 1) & 1]), ((blk - 1) >> 1) & 1, abort_flag));
         if (!ok) break;
       }
       tc_fence_after();

@@ -70,6 +70,18 @@ def test_append_kernels_agree(seed):
     assert np.max(np.abs(tc_lse - ms_lse)) <= 1e-3
 
 
+@pytest.mark.parametrize("window", [0, 128])
+def test_many_append_tiles_per_cta(window):
+    # thousands of append tiles: every persistent CTA runs many items in a row
+    rng = np.random.default_rng(700 + window)
+    B = 48
+    L = rng.integers(100, 260, size=B)
+    S = L + rng.integers(0, 900, size=B)
+    b = W.build_batch("manytiles", 800 + window, S, L, 64, 8, layer_windows=(window,))
+    run, _ = _full_check(b, what=f"manytiles w{window}")
+    assert run.header()["n_append"] * 8 > 20 * 152
+
+
 @pytest.mark.parametrize("split_pages", [1, 2, 3, 8, 1000])
 def test_split_length_does_not_change_results(split_pages):
     b = W.build_batch("splits", 55, [700, 33, 2049, 16, 1], [1, 1, 1, 1, 1], 32, 8)
