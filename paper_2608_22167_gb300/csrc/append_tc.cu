@@ -319,9 +319,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
         for (int c = 0; c < 4; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            mxa = fmaxf(mxa, __uint_as_float(sv[c][e]));
-            mxb = fmaxf(mxb, __uint_as_float(sv[c][e + 1]));
+          for (int e = 0; e < 32; e += 4) {
+            mxa = fmax3(mxa, __uint_as_float(sv[c][e]), __uint_as_float(sv[c][e + 1]));
+            mxb = fmax3(mxb, __uint_as_float(sv[c][e + 2]), __uint_as_float(sv[c][e + 3]));
           }
         const float mx = fmaxf(mxa, mxb) * p.scale_log2;
         float alpha = 1.f;
@@ -330,20 +330,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           m_ref = mx;
         }
         const float neg_mu = m_ref == -INFINITY ? 0.f : -m_ref;
-        const float sl2 = p.scale_log2;
-        float la = 0.f, lb = 0.f;
+        // p = 2^(s * scale * log2e - m): the argument in packed pairs
+        const uint64_t sl2x2 = pack_f32x2(p.scale_log2, p.scale_log2);
+        const uint64_t nmux2 = pack_f32x2(neg_mu, neg_mu);
+        uint64_t lsum = 0;  // two partial row sums
         uint32_t pk[2][32];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            const float p0 = ex2_approx(fmaf(__uint_as_float(sv[c][e]), sl2, neg_mu));
-            const float p1 = ex2_approx(fmaf(__uint_as_float(sv[c][e + 1]), sl2, neg_mu));
-            la += p0;
-            lb += p1;
+            const uint64_t x = fma2((uint64_t)sv[c][e] | ((uint64_t)sv[c][e + 1] << 32), sl2x2, nmux2);
+            const float p0 = ex2_approx(lo_f32(x));
+            const float p1 = ex2_approx(hi_f32(x));
+            lsum = add2(lsum, pack_f32x2(p0, p1));
             pk[c >> 1][(c & 1) * 16 + e / 2] = pack_bf16x2(p0, p1);
           }
         }
+        const float la = lo_f32(lsum), lb = hi_f32(lsum);
         l = l * alpha + (la + lb);
         // O may only be rescaled once PV_{blk-1} has completed. Without a
         // rescale P_blk is published right away: PV_blk queues behind
