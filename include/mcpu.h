@@ -142,6 +142,36 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
                                          float* lse, void* workspace, size_t workspace_bytes,
                                          const mcpu_options* opts, mcpu_stream_t stream);
 
+/*
+ * Paged attention forward for callers that cannot allocate device memory
+ * (an engine that reserves all GPU memory up front, code running under CUDA
+ * graph stream capture, a host that only receives device pointers). It has
+ * no counterpart in the paper: it is a deployment variant of
+ * mcpu_paged_attention_forward that takes no workspace. Its scratch (status
+ * word and work plan) lives in a 4 MiB array in the library's own device
+ * memory, held by every GPU that loads the library until the process exits.
+ *
+ * Same arguments and results as mcpu_paged_attention_forward (up to
+ * rounding), except:
+ *  - no workspace and no options: decode rows are not split across SMs and
+ *    the shared-prefix pass is off, so long decode rows run slower;
+ *  - total_q <= 262144 (num_seqs <= 2048 as for the other entry point);
+ *    larger batches return MCPU_ERR_WORKSPACE_TOO_SMALL without launching;
+ *  - `status_word` (device int32, may be NULL) receives this call's device
+ *    status bits (same meaning as the workspace status word), copied on
+ *    `stream` after the kernels.
+ * Every call on a device shares the one scratch array, which keeps the last
+ * call's contents (the call clears the status word itself): calls that
+ * overlap on the GPU (different streams, no ordering between them) race.
+ * The first call on a device looks up the array's device address and sets
+ * kernel attributes; make that first call before any stream capture.
+ */
+mcpu_status mcpu_paged_attention_forward_noalloc(const void* q, const void* k_cache, const void* v_cache,
+                                                 const int32_t* block_table, const int32_t* seq_lens,
+                                                 const int32_t* query_start_loc, int32_t sliding_window,
+                                                 float softmax_scale, const mcpu_dims* dims, void* out,
+                                                 float* lse, int32_t* status_word, mcpu_stream_t stream);
+
 /* Synchronises `stream`, reads the workspace status word and maps it to the
  * most severe mcpu_status (MCPU_OK if clear). The raw bits go to
  * *status_bits if non-NULL. The word is not cleared. */

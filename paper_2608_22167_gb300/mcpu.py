@@ -82,6 +82,10 @@ _lib.mcpu_paged_attention_forward.argtypes = [
     ctypes.POINTER(Options), _P,
 ]
 _lib.mcpu_paged_attention_forward.restype = ctypes.c_int
+_lib.mcpu_paged_attention_forward_noalloc.argtypes = [
+    _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P, _P,
+]
+_lib.mcpu_paged_attention_forward_noalloc.restype = ctypes.c_int
 _lib.mcpu_read_device_status.argtypes = [_P, _P, ctypes.POINTER(ctypes.c_int32)]
 _lib.mcpu_read_device_status.restype = ctypes.c_int
 _lib.mcpu_reset_device_status.argtypes = [_P, _P]
@@ -173,6 +177,21 @@ def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, que
             int(workspace.numel() * workspace.element_size()), ctypes.byref(opts), _stream(stream),
         ),
         "mcpu_paged_attention_forward",
+    )
+
+
+def mcpu_paged_attention_forward_noalloc(q, k_cache, v_cache, block_table, seq_lens, query_start_loc,
+                                         sliding_window, softmax_scale, out, lse, status_word=None, stream=None):
+    """The forward without a workspace (scratch in the library's own device
+    memory); status_word: optional device int32 tensor for the status bits."""
+    d = dims(q, k_cache, block_table, seq_lens)
+    _check(
+        _lib.mcpu_paged_attention_forward_noalloc(
+            _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc),
+            int(sliding_window), float(softmax_scale), ctypes.byref(d), _ptr(out), _ptr(lse), _ptr(status_word),
+            _stream(stream),
+        ),
+        "mcpu_paged_attention_forward_noalloc",
     )
 
 
