@@ -92,14 +92,17 @@ typedef struct mcpu_dims {
 /* Optional knobs of the forward pass; pass NULL for the defaults. */
 #define MCPU_FLAG_NO_CASCADE 0x1u       /* never run the shared-prefix (cascade) pass */
 #define MCPU_FLAG_MMA_SYNC_APPEND 0x2u  /* append chunks on the mma.sync kernel instead of tcgen05 */
+#define MCPU_FLAG_SERIAL 0x4u           /* run every kernel on `stream` (no side stream) */
 typedef struct mcpu_options {
   uint32_t flags;             /* MCPU_FLAG_* */
   int32_t split_pages;        /* > 0: KV split length of decode rows, in pages (0 = auto) */
   /* Optional timing hook: if non-NULL, MCPU_NUM_PHASE_EVENTS cudaEvent_t
-   * handles (created by the caller) that the call records on `stream`:
-   * [0] before the planner, [1] after it, [2] after the cascade pass,
-   * [3] after split-KV decode, [4] after the append-chunk kernel,
-   * [5] after the merge. Differences of consecutive events time each kernel. */
+   * handles (created by the caller) that the call records: [0] before the
+   * planner, [1] after it, [2] after split-KV decode, [3] after the cascade
+   * pass, [4] after the append-chunk kernel, [5] after the merge. By default
+   * decode and cascade run, in that order, on the library's side stream
+   * concurrently with the append kernel on `stream`: then [2] and [3] are
+   * recorded on the side stream and the append kernel spans [1]..[4]. */
   void* const* phase_events;
 } mcpu_options;
 #define MCPU_NUM_PHASE_EVENTS 6
@@ -134,6 +137,11 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
  * common full pages are read once for the whole group (full-context calls
  * only). Long decode rows are split over SMs and merged by log-sum-exp.
  * Results do not depend on the split or cascade choices beyond rounding.
+ * The memory-bound decode kernels run concurrently with the tensor-core
+ * append kernel: the call forks them onto a library-owned, low-priority
+ * stream of the current device after the planner and joins back before the
+ * merge, with CUDA events (this also works under stream capture). Pass
+ * MCPU_FLAG_SERIAL to keep every kernel on `stream`.
  */
 mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, const void* v_cache,
                                          const int32_t* block_table, const int32_t* seq_lens,

@@ -23,6 +23,8 @@ cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, c
                              const AttnParams& p, int grid, cudaStream_t stream);
 cudaError_t prepare_append_tc_kernel(int* bpsm);
 cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream);
+cudaError_t prepare_merge_kernel();
+cudaError_t prepare_kv_append_kernel();
 cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
                              const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
                              int32_t* status, int32_t num_seqs, int32_t total_q, int32_t max_pages,
@@ -39,6 +41,10 @@ struct DeviceState {
   bool ready = false;
   int sms = 0;
   int bpsm_decode = 0, bpsm_cascade = 0, bpsm_append = 0, bpsm_append_tc = 0;
+  // side stream for the memory-bound decode kernels, and the fork/join events
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  std::mutex fork_mu;  // one fork/join sequence at a time per device
 };
 
 std::mutex g_mu;
@@ -66,8 +72,15 @@ mcpu_status device_state(DeviceState** out) {
     if (prepare_decode_kernels(&st.bpsm_decode, &st.bpsm_cascade) != cudaSuccess) return MCPU_ERR_CUDA;
     if (prepare_append_kernel(&st.bpsm_append) != cudaSuccess) return MCPU_ERR_CUDA;
     if (prepare_append_tc_kernel(&st.bpsm_append_tc) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (prepare_merge_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
+    if (prepare_kv_append_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
     if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1 || st.bpsm_append_tc < 1)
       return MCPU_ERR_CUDA;
+    int lo_prio = 0, hi_prio = 0;
+    if (cudaDeviceGetStreamPriorityRange(&lo_prio, &hi_prio) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (cudaStreamCreateWithPriority(&st.side, cudaStreamNonBlocking, lo_prio) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (cudaEventCreateWithFlags(&st.ev_fork, cudaEventDisableTiming) != cudaSuccess) return MCPU_ERR_CUDA;
+    if (cudaEventCreateWithFlags(&st.ev_join, cudaEventDisableTiming) != cudaSuccess) return MCPU_ERR_CUDA;
     st.ready = true;
   }
   *out = &st;
@@ -160,6 +173,9 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
       !aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(query_start_loc, 4) || !aligned(status_word, 4))
     return MCPU_ERR_INVALID_ARG;
   if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  DeviceState* dev = nullptr;  // one-time per-device kernel setup
+  st = device_state(&dev);
+  if (st != MCPU_OK) return st;
   return from_cuda(launch_kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start_loc,
                                     status_word, dims->num_seqs, dims->total_q, dims->max_pages_per_seq,
                                     dims->num_pages, dims->num_kv_heads, reinterpret_cast<cudaStream_t>(stream)));
@@ -222,30 +238,51 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   void* const* ev = opts ? opts->phase_events : nullptr;
-  auto mark = [&](int i) -> cudaError_t {
-    return ev ? cudaEventRecord(reinterpret_cast<cudaEvent_t>(ev[i]), s) : cudaSuccess;
+  auto mark = [&](int i, cudaStream_t on) -> cudaError_t {
+    return ev ? cudaEventRecord(reinterpret_cast<cudaEvent_t>(ev[i]), on) : cudaSuccess;
   };
-  cudaError_t e = mark(0);
+  const bool serial = opts && (opts->flags & MCPU_FLAG_SERIAL);
+  const bool cascade = p.cascade_enabled && p.window == 0;
+  auto launch_append_kernel = [&]() -> cudaError_t {
+    if (legacy_append) return launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
+    return launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
+  };
+  cudaError_t e = mark(0, s);
   if (e == cudaSuccess) e = launch_plan(p, s);
-  if (e == cudaSuccess) e = mark(1);
-  if (e == cudaSuccess && p.cascade_enabled && p.window == 0)
-    e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, s);
-  if (e == cudaSuccess) e = mark(2);
-  if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s);
-  if (e == cudaSuccess) e = mark(3);
-  if (e == cudaSuccess) {
-    if (legacy_append)
-      e = launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
-    else
-      e = launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
+  if (e == cudaSuccess) e = mark(1, s);
+  if (serial) {
+    if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s);
+    if (e == cudaSuccess) e = mark(2, s);
+    if (e == cudaSuccess && cascade) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, s);
+    if (e == cudaSuccess) e = mark(3, s);
+    if (e == cudaSuccess) e = launch_append_kernel();
+    if (e == cudaSuccess) e = mark(4, s);
+  } else {
+    // fork: the append kernel goes first on `stream` (its CTAs claim the
+    // SMs); the decode kernel follows on the low-priority side stream and its
+    // CTAs (few registers) fill the room each SM has left. The cascade pass
+    // comes after decode on the side stream: its CTAs need more registers
+    // than an SM running an append CTA has free, so it may only start as the
+    // append kernel drains. Join before the merge.
+    std::lock_guard<std::mutex> lock(dev->fork_mu);
+    if (e == cudaSuccess) e = cudaEventRecord(dev->ev_fork, s);
+    if (e == cudaSuccess) e = launch_append_kernel();
+    if (e == cudaSuccess) e = mark(4, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(dev->side, dev->ev_fork, 0);
+    if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, dev->side);
+    if (e == cudaSuccess) e = mark(2, dev->side);
+    if (e == cudaSuccess && cascade)
+      e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, dev->side);
+    if (e == cudaSuccess) e = mark(3, dev->side);
+    if (e == cudaSuccess) e = cudaEventRecord(dev->ev_join, dev->side);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, dev->ev_join, 0);
   }
-  if (e == cudaSuccess) e = mark(4);
   if (e == cudaSuccess) {
     const int want = (p.num_seqs * p.num_q_heads + 7) / 8;
     const int grid = want < dev->sms * 8 ? (want > 0 ? want : 1) : dev->sms * 8;
     e = launch_merge(p, grid, s);
   }
-  if (e == cudaSuccess) e = mark(5);
+  if (e == cudaSuccess) e = mark(5, s);
   return from_cuda(e);
 }
 

@@ -258,6 +258,9 @@ cudaError_t prepare_append_kernel(int* blocks_per_sm) {
   cudaError_t e = cudaFuncSetAttribute(append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)append_smem_bytes());
   if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(append_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_kernel, kAppWarps * 32,
                                                        append_smem_bytes());
 }

@@ -432,6 +432,9 @@ cudaError_t prepare_append_tc_kernel(int* blocks_per_sm) {
   cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)append_tc_smem_bytes());
   if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_tc_kernel, kTcThreads,
                                                        append_tc_smem_bytes());
 }

@@ -65,8 +65,10 @@ struct PlanHeader {
   int32_t n_merge;       // MergeRow records
   int32_t split_pages;   // chosen split length, for inspection
   int32_t n_parts;       // partial slots in use
-  int32_t append_ticket; // dynamic scheduler counter of the append kernel
-  int32_t pad[56];
+  int32_t append_ticket; // dynamic scheduler counters, reset by the planner
+  int32_t decode_ticket;
+  int32_t cascade_ticket;
+  int32_t pad[54];
 };
 static_assert(sizeof(PlanHeader) == 256, "header is one 256-byte block");
 

@@ -14,7 +14,7 @@
 //     O^T += V^T P^T (head dim as M) in fp32.
 // The item ends with either the final bf16 output + lse (a decode row that
 // needs one split) or a normalised fp32 partial + base-2 lse in a workspace
-// slot, merged later by log-sum-exp.
+// slot, merged later by log-sum-exp. Warps take items from an atomic ticket.
 //
 // HBM traffic per (page, kv head): 4 KiB read once. Nothing else is re-read.
 #include "common.cuh"
@@ -62,8 +62,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
   const uint64_t pol = policy_evict_first();
   const int mi = lane >> 3, ri = lane & 7;
 
+  // Items are taken from an atomic ticket, one per warp at a time, so warps
+  // that start late (their SM busy with another kernel) take fewer items.
+  int* ticket = NT == 1 ? &header(p)->decode_ticket : &header(p)->cascade_ticket;
+  auto next_item = [&]() -> int {
+    int v = 0;
+    if (lane == 0) v = atomicAdd(ticket, 1);
+    return __shfl_sync(0xffffffffu, v, 0);
+  };
   uint32_t seq = 0;  // pages this warp has consumed so far (ring position/phase)
-  for (int it = blockIdx.x * kDecodeWarps + warp; it < n_items; it += gridDim.x * kDecodeWarps) {
+  for (int it = next_item(); it < n_items; it = next_item()) {
     const int rec = it / Hkv, kvh = it % Hkv;
     int row, pb, pe, seq_len = 0, first_key = 0, slot = -1, token = 0;
     int member_off = 0, n_members = 0, split = 0;
@@ -310,6 +318,14 @@ cudaError_t prepare_decode_kernels(int* blocks_per_sm_decode, int* blocks_per_sm
   e = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decode_smem_bytes());
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(decode_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decode_smem_bytes());
+  if (e != cudaSuccess) return e;
+  // the same (largest) shared-memory carveout as the append kernel, so that
+  // decode CTAs can share an SM with an append CTA
+  e = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(decode_kernel<4>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
   if (e != cudaSuccess) return e;
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm_decode, decode_kernel<1>, kDecodeWarps * 32,
                                                     decode_smem_bytes());

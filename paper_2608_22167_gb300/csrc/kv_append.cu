@@ -78,6 +78,11 @@ __global__ void __launch_bounds__(kKvAppendThreads) kv_append_kernel(const KvApp
   }
 }
 
+cudaError_t prepare_kv_append_kernel() {
+  return cudaFuncSetAttribute(kv_append_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
+}
+
 cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
                              const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
                              int32_t* status, int32_t num_seqs, int32_t total_q, int32_t max_pages,

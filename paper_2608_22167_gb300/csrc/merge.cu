@@ -43,6 +43,11 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
   }
 }
 
+cudaError_t prepare_merge_kernel() {
+  return cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
+}
+
 cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream) {
   merge_kernel<<<grid, kMergeWarps * 32, 0, stream>>>(p);
   return cudaGetLastError();

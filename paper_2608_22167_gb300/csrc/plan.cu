@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     if (tid == 0) {
       hdr->n_decode = hdr->n_cascade = hdr->n_append = hdr->n_merge = 0;
       hdr->n_parts = 0;
-      hdr->append_ticket = 0;
+      hdr->append_ticket = hdr->decode_ticket = hdr->cascade_ticket = 0;
     }
     return;
   }
@@ -174,17 +174,29 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
       const int lim = min(sa, sb) / kPage;  // pages full in both rows
       const int* ba = p.block_table + (size_t)(r - 1) * p.max_pages;
       const int* bb = p.block_table + (size_t)r * p.max_pages;
+      // 128 entries per step: four independent loads per lane, then ballots
       int n = 0;
-      for (int base = 0; base < lim; base += 32) {
-        const int i = base + lane;
-        const bool eq = i < lim && __ldg(ba + i) == __ldg(bb + i);
-        const unsigned m = __ballot_sync(0xffffffffu, eq);
-        if (m == 0xffffffffu) {
-          n += 32;
-          continue;
+      for (int base = 0; base < lim; base += 128) {
+        bool eq[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int i = base + 32 * j + lane;
+          eq[j] = i < lim && __ldg(ba + i) == __ldg(bb + i);
         }
-        n += __ffs(~m) - 1;
-        break;
+        bool stop = false;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const unsigned m = __ballot_sync(0xffffffffu, eq[j]);
+          if (!stop) {
+            if (m == 0xffffffffu) {
+              n += 32;
+            } else {
+              n += __ffs(~m) - 1;
+              stop = true;
+            }
+          }
+        }
+        if (stop) break;
       }
       if (lane == 0) sm.lcp[r] = min(n, lim);
     }
@@ -320,7 +332,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
       atomicOr(&hdr->status, kStatusPlanOverflow);
       hdr->n_decode = hdr->n_cascade = hdr->n_append = hdr->n_merge = 0;
       hdr->n_parts = 0;
-      hdr->append_ticket = 0;
+      hdr->append_ticket = hdr->decode_ticket = hdr->cascade_ticket = 0;
     }
     return;
   }
@@ -414,7 +426,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     hdr->n_merge = is_merge_cnt;
     hdr->split_pages = C;
     hdr->n_parts = tot_parts;
-    hdr->append_ticket = 0;
+    hdr->append_ticket = hdr->decode_ticket = hdr->cascade_ticket = 0;
   }
 }
 
@@ -425,7 +437,13 @@ cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream) {
 }
 
 cudaError_t prepare_plan_kernel() {
-  return cudaFuncSetAttribute(plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(PlanSmem));
+  cudaError_t e = cudaFuncSetAttribute(plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(PlanSmem));
+  if (e != cudaSuccess) return e;
+  // every kernel of the library asks for the largest shared-memory carveout,
+  // so an SM never has to be reconfigured between them and a decode CTA can
+  // share an SM with an append CTA
+  return cudaFuncSetAttribute(plan_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
 }
 
 }  // namespace mcpu

@@ -82,6 +82,20 @@ def test_many_append_tiles_per_cta(window):
     assert run.header()["n_append"] * 8 > 20 * 152
 
 
+def test_side_stream_and_serial_orders_agree_bitwise():
+    # decode kernels on the library's side stream (default) or all on one stream
+    rng = np.random.default_rng(41)
+    S = rng.integers(1, 5000, size=20)
+    L = np.where(np.arange(20) % 4 == 0, np.minimum(S, rng.integers(2, 300, size=20)), 1)
+    b = W.build_batch("sides", 42, S, L, 64, 8)
+    run, _ = _full_check(b, what="side stream")
+    out1, lse1 = run.out_host()
+    run.forward(flags=mcpu.FLAG_SERIAL)
+    assert run.status()[0] == 0
+    out2, lse2 = run.out_host()
+    assert np.array_equal(out1, out2) and np.array_equal(lse1, lse2)
+
+
 @pytest.mark.parametrize("split_pages", [1, 2, 3, 8, 1000])
 def test_split_length_does_not_change_results(split_pages):
     b = W.build_batch("splits", 55, [700, 33, 2049, 16, 1], [1, 1, 1, 1, 1], 32, 8)
