@@ -61,6 +61,32 @@ WORKLOAD_DESC = {
 }
 
 
+def recorded_traffic(kernel_md: str, key: str, sources):
+    """DRAM bytes per launch recorded in a profiles/ summary, or None when the
+    kernel's sources changed since the capture (sha256 mismatch)."""
+    import hashlib
+    import re
+
+    path = os.path.join(ROOT, "profiles", kernel_md)
+    try:
+        text = open(path).read()
+        h = hashlib.sha256()
+        for f in sources:
+            h.update(open(os.path.join(ROOT, f), "rb").read())
+        sha = re.search(r"source_sha256: ([0-9a-f]{64})", text).group(1)
+        val = re.search(key + r": (\d+)", text).group(1)
+        return int(val) if sha == h.hexdigest() else None
+    except Exception:
+        return None
+
+
+APPEND_TC_SOURCES = [
+    "paper_2608_22167_gb300/csrc/append_tc.cu",
+    "paper_2608_22167_gb300/csrc/tcgen05.cuh",
+    "paper_2608_22167_gb300/csrc/common.cuh",
+]
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -384,8 +410,16 @@ def run_ours(args, rank, world, dev):
     roof_app = None
     if app_ms > 0 and app_flops > 0:
         ach = app_flops / (app_ms * 1e-3) / 1e12
+        traffic = None
+        if args.workload == "mixed":
+            traffic = recorded_traffic("append_tc_kernel_mixed.md", "traffic_bytes_per_launch_mixed",
+                                       APPEND_TC_SOURCES)
         roof_app = {"bound": "tensor", "achieved": round(ach, 2), "peak": tc_burst, "unit": "TFLOP/s",
-                    "frac": round(ach / tc_burst, 4), "traffic": None, "kernel": "append_kernel",
+                    "frac": round(ach / tc_burst, 4), "traffic": traffic,
+                    "algorithmic_bytes": int(sum(s["kv_bytes_append"] for s in per_layer)
+                                             + 2 * int(batch.q_lens[batch.q_lens > 1].sum()) * batch.num_q_heads
+                                             * batch.head_dim * 2),
+                    "kernel": "append_tc_kernel",
                     "peak_source": f"{peak_src} bf16_tflops (burst)", "ms_per_step": round(app_ms, 4)}
     cands = [r for r in (roof_dec, roof_app) if r is not None]
     dominant = max(cands, key=lambda r: r["ms_per_step"]) if cands else None
