@@ -85,6 +85,10 @@ APPEND_TC_SOURCES = [
     "paper_2608_22167_gb300/csrc/tcgen05.cuh",
     "paper_2608_22167_gb300/csrc/common.cuh",
 ]
+DECODE_SOURCES = [
+    "paper_2608_22167_gb300/csrc/decode.cu",
+    "paper_2608_22167_gb300/csrc/common.cuh",
+]
 
 
 def peaks():
@@ -347,14 +351,29 @@ def run_ours(args, rank, world, dev):
 
     nl = len(batch.layers)
     stream = torch.cuda.current_stream()
+    # one set of phase events per recorded step: every timed step in eager
+    # mode; in graph mode one set per captured graph (each graph records its
+    # own set at every replay, so the sets hold the graphs' last replays)
+    n_sets = args.steps if args.launch == "eager" else min(args.steps, 16)
     phase = [[[torch.cuda.Event(enable_timing=True) for _ in range(mcpu.NUM_PHASE_EVENTS)] for _ in range(nl)]
-             for _ in range(args.steps)]
+             for _ in range(n_sets)]
     for s in phase:  # create the events (torch creates them lazily)
         for lay in s:
             for e in lay:
                 e.record(stream)
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    graphs = []
+    if args.launch == "graph":
+        # the whole step (every layer's KV append and forward) as CUDA graphs;
+        # the planner runs inside the graph, so nothing is precomputed
+        for j in range(n_sets):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                st.step(events=phase[j])
+            graphs.append(g)
+        for g in graphs:  # upload, untimed
+            g.replay()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
     uuid = None
     try:
         uuid = str(torch.cuda.get_device_properties(dev).uuid)
@@ -368,34 +387,63 @@ def run_ours(args, rank, world, dev):
     sampler.start()
     time.sleep(0.3)  # let the sampler start before the timed region
     wall0 = time.perf_counter()
+    t_start.record(stream)
     for k in range(args.steps):
-        starts[k].record(stream)
-        st.step(events=phase[k])
-        ends[k].record(stream)
+        if graphs:
+            graphs[k % n_sets].replay()
+        else:
+            st.step(events=phase[k])
+    t_end.record(stream)
     torch.cuda.synchronize()
     wall = time.perf_counter() - wall0
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     clocks = sampler.stop()
-    step_ms = [starts[k].elapsed_time(ends[k]) for k in range(args.steps)]
-    total_ms = float(sum(step_ms))
+    total_ms = float(t_start.elapsed_time(t_end))
     code, bits = mcpu.mcpu_read_device_status(st.ws)
     if code != 0:
         raise RuntimeError(f"device status {bits} in the timed region")
 
+    # the other launch mode, same steps, for comparison (untimed for `value`)
+    other_ms = None
+    if args.compare_launch:
+        torch.cuda.synchronize()
+        o0 = torch.cuda.Event(enable_timing=True)
+        o1 = torch.cuda.Event(enable_timing=True)
+        n_other = min(args.steps, 50)
+        if graphs:
+            o0.record(stream)
+            for k in range(n_other):
+                st.step()
+            o1.record(stream)
+        else:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                st.step()
+            g.replay()
+            o0.record(stream)
+            for k in range(n_other):
+                g.replay()
+            o1.record(stream)
+        torch.cuda.synchronize()
+        other_ms = o0.elapsed_time(o1) / n_other
+
     # per-kernel times, ms per step. Decode then cascade run on the library's
     # side stream concurrently with the append kernel: events [1]->[2]
-    # decode, [2]->[3] cascade (side stream), [1]->[4] append, [4]->[5] merge
-    # (after the join, so it includes waiting for the side stream).
-    spans = {"plan": (0, 1), "decode": (1, 2), "cascade": (2, 3), "append_chunk": (1, 4), "merge": (4, 5)}
-    ktime = {n: 0.0 for n in spans}
-    for k in range(args.steps):
+    # decode, [2]->[3] cascade (side stream), [1]->[4] append; the merge
+    # starts at the join, the later of [3] and [4].
+    ktime = {n: 0.0 for n in ("plan", "decode", "cascade", "append_chunk", "merge")}
+    for k in range(n_sets):
         for i in range(nl):
             ev = phase[k][i]
-            for n, (a, b_) in spans.items():
-                ktime[n] += ev[a].elapsed_time(ev[b_])
-    ktime = {n: v / args.steps for n, v in ktime.items()}
+            t = [0.0] + [ev[0].elapsed_time(ev[j]) for j in range(1, len(ev))]
+            ktime["plan"] += t[1]
+            ktime["decode"] += t[2] - t[1]
+            ktime["cascade"] += t[3] - t[2]
+            ktime["append_chunk"] += t[4] - t[1]
+            ktime["merge"] += t[5] - max(t[3], t[4])
+    ktime = {n: v / n_sets for n, v in ktime.items()}
     dec_bytes = sum(s["kv_bytes"] - s["kv_bytes_append"] for s in per_layer)
     app_flops = sum(s["flops_append"] for s in per_layer)
     dec_ms = ktime["cascade"] + ktime["decode"]
@@ -403,8 +451,12 @@ def run_ours(args, rank, world, dev):
     roof_dec = None
     if dec_ms > 0 and dec_bytes > 0:
         ach = dec_bytes / (dec_ms * 1e-3) / 1e9
+        traffic = None
+        if args.workload in ("decode", "long"):
+            traffic = recorded_traffic("decode_kernel_decode_long.md", f"traffic_bytes_per_launch_{args.workload}",
+                                       DECODE_SOURCES)
         roof_dec = {"bound": "hbm", "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
-                    "frac": round(ach / hbm, 4), "traffic": None,
+                    "frac": round(ach / hbm, 4), "traffic": traffic,
                     "kernel": "decode_kernel (+cascade pass)", "peak_source": f"{peak_src} hbm_gbs",
                     "ms_per_step": round(dec_ms, 4)}
     roof_app = None
@@ -501,10 +553,13 @@ def run_ours(args, rank, world, dev):
             "l2": "inputs larger than L2 (KV pool %.1f GB >> 126 MB L2); no flush" % (
                 sum(p.k_cache.numel() * 4 for p in batch.pools.values()) / 1e9),
             "parallelism": f"replicas x{world} (no exchange step)",
+            "launch": "one CUDA graph per step (KV append + forward of every layer)" if graphs
+                      else "eager (C-ABI calls per layer)",
         },
         "frac_of_hbm_peak": round(value / world / hbm, 4),
         "attended_tokens_per_s": round(pairs * world / (ms_per_step * 1e-3), 1),
         "kernel_ms_per_step": {k: round(v, 4) for k, v in ktime.items()},
+        ("eager_ms_per_step" if graphs else "graph_ms_per_step"): (round(other_ms, 4) if other_ms else None),
         "roofline": dominant,
         "roofline_decode": roof_dec,
         "roofline_append": roof_app,
@@ -569,6 +624,10 @@ def main():
     ap.add_argument("--workload", choices=sorted(W.CONFIGS), default="mixed")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--launch", choices=["graph", "eager"], default="eager",
+                    help="time eager C-ABI calls (default) or CUDA-graph replays of the whole step")
+    ap.add_argument("--no-compare-launch", dest="compare_launch", action="store_false",
+                    help="skip timing the other launch mode")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

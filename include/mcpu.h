@@ -102,7 +102,9 @@ typedef struct mcpu_options {
    * pass, [4] after the append-chunk kernel, [5] after the merge. By default
    * decode and cascade run, in that order, on the library's side stream
    * concurrently with the append kernel on `stream`: then [2] and [3] are
-   * recorded on the side stream and the append kernel spans [1]..[4]. */
+   * recorded on the side stream and the append kernel spans [1]..[4].
+   * Under stream capture they become event-record nodes of the graph, so
+   * every replay records them. */
   void* const* phase_events;
 } mcpu_options;
 #define MCPU_NUM_PHASE_EVENTS 6
@@ -140,8 +142,14 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
  * The memory-bound decode kernels run concurrently with the tensor-core
  * append kernel: the call forks them onto a library-owned, low-priority
  * stream of the current device after the planner and joins back before the
- * merge, with CUDA events (this also works under stream capture). Pass
- * MCPU_FLAG_SERIAL to keep every kernel on `stream`.
+ * merge, with CUDA events. Pass MCPU_FLAG_SERIAL to keep every kernel on
+ * `stream`. The call is capturable in a CUDA graph (with mcpu_kv_append
+ * before it): it allocates nothing, synchronises nothing, and its work plan
+ * is rebuilt on the device at every replay, so a replayed graph follows
+ * changed seq_lens / block_table / query_start_loc contents as long as the
+ * dims (and hence the pointers' extents) stay the same. The first call on a
+ * device sets kernel attributes and creates the side stream; make it before
+ * any capture.
  */
 mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, const void* v_cache,
                                          const int32_t* block_table, const int32_t* seq_lens,
@@ -190,6 +198,12 @@ mcpu_status mcpu_reset_device_status(void* workspace, mcpu_stream_t stream);
 
 /* Static, human-readable name of a status code. */
 const char* mcpu_status_string(mcpu_status status);
+
+/* The cudaError_t (as an integer) of the most recent CUDA call that failed
+ * inside mcpu_kv_append or mcpu_paged_attention_forward on the calling
+ * thread, i.e. the cause behind their last MCPU_ERR_CUDA; 0 if none has
+ * failed. Not cleared by later successful calls. */
+int32_t mcpu_last_cuda_error(void);
 
 /* Version of this ABI (bumped on any signature change). */
 int32_t mcpu_abi_version(void);

@@ -50,11 +50,21 @@ struct DeviceState {
 std::mutex g_mu;
 DeviceState g_dev[kMaxDevices];
 
+// most recent failing CUDA call of this thread's entry-point calls
+thread_local int32_t t_last_cuda_error = 0;
+
+mcpu_status cuda_fail(cudaError_t e) {
+  t_last_cuda_error = (int32_t)e;
+  return MCPU_ERR_CUDA;
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 mcpu_status device_state(DeviceState** out) {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MCPU_ERR_CUDA;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= kMaxDevices) return MCPU_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_mu);
   DeviceState& st = g_dev[dev];
   if (!st.ready) {
@@ -67,20 +77,20 @@ mcpu_status device_state(DeviceState** out) {
         return MCPU_ERR_CUDA;
       g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
-    if (cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_plan_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_decode_kernels(&st.bpsm_decode, &st.bpsm_cascade) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_append_kernel(&st.bpsm_append) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_append_tc_kernel(&st.bpsm_append_tc) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_merge_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_kv_append_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
+    if ((e = cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_plan_kernel()) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_decode_kernels(&st.bpsm_decode, &st.bpsm_cascade)) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_append_kernel(&st.bpsm_append)) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_append_tc_kernel(&st.bpsm_append_tc)) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_merge_kernel()) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_kv_append_kernel()) != cudaSuccess) return cuda_fail(e);
     if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1 || st.bpsm_append_tc < 1)
       return MCPU_ERR_CUDA;
     int lo_prio = 0, hi_prio = 0;
-    if (cudaDeviceGetStreamPriorityRange(&lo_prio, &hi_prio) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (cudaStreamCreateWithPriority(&st.side, cudaStreamNonBlocking, lo_prio) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (cudaEventCreateWithFlags(&st.ev_fork, cudaEventDisableTiming) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (cudaEventCreateWithFlags(&st.ev_join, cudaEventDisableTiming) != cudaSuccess) return MCPU_ERR_CUDA;
+    if ((e = cudaDeviceGetStreamPriorityRange(&lo_prio, &hi_prio)) != cudaSuccess) return cuda_fail(e);
+    if ((e = cudaStreamCreateWithPriority(&st.side, cudaStreamNonBlocking, lo_prio)) != cudaSuccess) return cuda_fail(e);
+    if ((e = cudaEventCreateWithFlags(&st.ev_fork, cudaEventDisableTiming)) != cudaSuccess) return cuda_fail(e);
+    if ((e = cudaEventCreateWithFlags(&st.ev_join, cudaEventDisableTiming)) != cudaSuccess) return cuda_fail(e);
     st.ready = true;
   }
   *out = &st;
@@ -132,13 +142,15 @@ mcpu_status check_dims(const mcpu_dims* d) {
   return MCPU_OK;
 }
 
-mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : MCPU_ERR_CUDA; }
+mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : cuda_fail(e); }
 
 }  // namespace
 
 extern "C" {
 
 int32_t mcpu_abi_version(void) { return 1; }
+
+int32_t mcpu_last_cuda_error(void) { return t_last_cuda_error; }
 
 const char* mcpu_status_string(mcpu_status s) {
   switch (s) {
@@ -238,8 +250,16 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   void* const* ev = opts ? opts->phase_events : nullptr;
+  // Under stream capture the phase events become event-record nodes of the
+  // graph (recorded at every replay); otherwise plain event records.
+  cudaStreamCaptureStatus capturing = cudaStreamCaptureStatusNone;
+  if (ev) {
+    const cudaError_t ce = cudaStreamIsCapturing(reinterpret_cast<cudaStream_t>(stream), &capturing);
+    if (ce != cudaSuccess) return cuda_fail(ce);
+  }
+  const unsigned int rec_flags = capturing == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : 0u;
   auto mark = [&](int i, cudaStream_t on) -> cudaError_t {
-    return ev ? cudaEventRecord(reinterpret_cast<cudaEvent_t>(ev[i]), on) : cudaSuccess;
+    return ev ? cudaEventRecordWithFlags(reinterpret_cast<cudaEvent_t>(ev[i]), on, rec_flags) : cudaSuccess;
   };
   const bool serial = opts && (opts->flags & MCPU_FLAG_SERIAL);
   const bool cascade = p.cascade_enabled && p.window == 0;

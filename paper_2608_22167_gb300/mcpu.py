@@ -50,6 +50,8 @@ class McpuError(RuntimeError):
         self.code = code
         name = STATUS.get(code, str(code))
         msg = _lib.mcpu_status_string(code).decode()
+        if code == 4:
+            msg += f", cudaError_t {int(_lib.mcpu_last_cuda_error())}"
         super().__init__(f"{where}: {name} ({msg})")
 
 
@@ -95,6 +97,8 @@ _lib.mcpu_status_string.argtypes = [ctypes.c_int]
 _lib.mcpu_status_string.restype = ctypes.c_char_p
 _lib.mcpu_abi_version.argtypes = []
 _lib.mcpu_abi_version.restype = ctypes.c_int32
+_lib.mcpu_last_cuda_error.argtypes = []
+_lib.mcpu_last_cuda_error.restype = ctypes.c_int32
 
 
 def _ptr(t):
@@ -129,6 +133,10 @@ def dims(q, k_cache, block_table, seq_lens) -> Dims:
 
 def mcpu_abi_version() -> int:
     return int(_lib.mcpu_abi_version())
+
+
+def mcpu_last_cuda_error() -> int:
+    return int(_lib.mcpu_last_cuda_error())
 
 
 def mcpu_status_string(code: int) -> str:
@@ -169,6 +177,9 @@ def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, que
     opts = Options(flags=int(flags), split_pages=int(split_pages), phase_events=None)
     if phase_events is not None:
         assert len(phase_events) == NUM_PHASE_EVENTS
+        if any(e.cuda_event == 0 for e in phase_events):
+            raise ValueError("torch creates a CUDA event at its first record(): record each phase event once "
+                             "before passing it")
         arr = (ctypes.c_void_p * NUM_PHASE_EVENTS)(*[ctypes.c_void_p(e.cuda_event) for e in phase_events])
         opts.phase_events = ctypes.cast(arr, ctypes.c_void_p)
     _check(

@@ -223,3 +223,58 @@ def test_rollout_step_sampled_every_layer():
         _sampled_check(b, rows, n_per_row=6, seed=100 + layer, layer=layer, run=run)
         del run
         torch.cuda.empty_cache()
+
+
+# ------------------------------------------------------------ CUDA graphs
+
+
+def test_cuda_graph_replay_follows_new_lengths():
+    # KV append + forward captured once; the planner runs inside the graph, so
+    # a replay after seq_lens changed (same dims) computes the new batch
+    import dataclasses
+
+    rng = np.random.default_rng(61)
+    B = 12
+    S = rng.integers(200, 3000, size=B)
+    L = np.where(np.arange(B) % 3 == 0, np.minimum(S - 150, rng.integers(2, 300, size=B)), 1)
+    b = W.build_batch("graph", 62, S, L, 64, 8)
+    run = Run(b)
+    k0, v0 = run.kc.clone(), run.vc.clone()
+    run.append()
+    run.forward()
+    assert run.status()[0] == 0
+    out_e, lse_e = run.out_host()
+
+    run.kc.copy_(k0)
+    run.vc.copy_(v0)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(mcpu.NUM_PHASE_EVENTS)]
+    for e in ev:  # torch creates the CUDA event at its first record
+        e.record()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        run.append()
+        mcpu.mcpu_paged_attention_forward(run.q, run.kc, run.vc, run.bt, run.sl, run.qsl, run.window,
+                                          b.softmax_scale, run.out, run.lse, run.ws, phase_events=ev)
+    run.out.fill_(float("nan"))
+    g.replay()
+    assert run.status()[0] == 0
+    out_g, lse_g = run.out_host()
+    assert np.array_equal(out_g, out_e) and np.array_equal(lse_g, lse_e)
+    assert ev[0].elapsed_time(ev[5]) > 0  # the phase events are graph nodes
+
+    # shorter contexts, same chunks and pages: replay the same graph
+    S2 = (S - rng.integers(1, 150, size=B)).astype(np.int32)
+    b2 = dataclasses.replace(b, seq_lens=S2)
+    run.kc.copy_(k0)
+    run.vc.copy_(v0)
+    run.sl.copy_(torch.from_numpy(S2))
+    run.out.fill_(float("nan"))
+    g.replay()
+    assert run.status()[0] == 0
+    ref_out, ref_lse, (okc, ovc) = oracle_full(b2)
+    assert np.array_equal(W.to_host(run.kc), okc) and np.array_equal(W.to_host(run.vc), ovc)
+    got_out, got_lse = run.out_host()
+    assert_parity(got_out, got_lse, ref_out, ref_lse, "graph replay, new lengths")
+    assert np.abs(got_out - out_e).max() > 0  # the replay did compute the new batch
