@@ -110,12 +110,13 @@ bool encode_pool(CUtensorMap* map, const void* pool, int64_t rows) {
   return r == CUDA_SUCCESS;
 }
 
-// 3-D view of q [T, H_q, D]: boxes of (128 / g) tokens x the g heads of one kv
-// head x 64 dims, i.e. one 128-row query tile, 128-byte swizzle.
+// 3-D view of q [T, H_q, D]: boxes of (256 / g) tokens x the g heads of one kv
+// head x 64 dims, i.e. the two 128-row query tiles of an append item, 128-byte
+// swizzle.
 bool encode_query(CUtensorMap* map, const void* q, int32_t total_q, int32_t num_q_heads, int32_t group) {
   cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)num_q_heads, (cuuint64_t)total_q};
   cuuint64_t strides[2] = {(cuuint64_t)kRowBytes, (cuuint64_t)kRowBytes * num_q_heads};
-  cuuint32_t box[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)group, (cuuint32_t)(128 / group)};
+  cuuint32_t box[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)group, (cuuint32_t)(kAppendTcRows / group)};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -246,7 +247,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   p.forced_split_pages = opts ? opts->split_pages : 0;
   p.cascade_enabled = (opts && (opts->flags & MCPU_FLAG_NO_CASCADE)) ? 0 : 1;
   p.oob_row = (int32_t)rows;
-  p.append_tile_tok = (legacy_append ? kAppendRowsMin : 128) / p.group;
+  p.append_tile_tok = (legacy_append ? kAppendRowsMin : kAppendTcRows) / p.group;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   void* const* ev = opts ? opts->phase_events : nullptr;

@@ -143,7 +143,7 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
     const cuuint32_t pbox[2] = {(cuuint32_t)kHeadDim, (cuuint32_t)kPage};
     const cuuint64_t qdims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)d.num_q_heads, (cuuint64_t)d.total_q};
     const cuuint64_t qstr[2] = {(cuuint64_t)kRowBytes, (cuuint64_t)kRowBytes * d.num_q_heads};
-    const cuuint32_t qbox[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)group, (cuuint32_t)(128 / group)};
+    const cuuint32_t qbox[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)group, (cuuint32_t)(kAppendTcRows / group)};
     if (!encode_tiled(&kmap, k_cache, 2, pdims, pstr, pbox) || !encode_tiled(&vmap, v_cache, 2, pdims, pstr, pbox) ||
         !encode_tiled(&qmap, q, 3, qdims, qstr, qbox))
       return MCPU_ERR_INVALID_ARG;
@@ -171,7 +171,7 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
   p.forced_split_pages = 0x3fffffff;  // one split per decode row: every row writes out/lse itself
   p.cascade_enabled = 0;
   p.oob_row = (int32_t)rows;
-  p.append_tile_tok = 128 / group;
+  p.append_tile_tok = kAppendTcRows / group;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // The scratch keeps the previous call's contents: the status word must

@@ -25,6 +25,7 @@ constexpr int kSplitBudget = 4096;    // bound on member-weighted KV splits per 
 constexpr int kMinSplitPages = 8;     // shortest split of a decode row, in pages
 constexpr int kMinSharedPages = 4;    // shortest prefix worth a cascade pass
 constexpr int kAppendRowsMin = 64;    // smallest append tile (query rows = tokens x heads)
+constexpr int kAppendTcRows = 256;    // query rows of one tcgen05 append item (two 128-row tiles)
 
 // Status bits, OR-ed into the first word of the workspace. They are sticky
 // until the caller resets them.

@@ -74,8 +74,8 @@ def test_append_kernels_agree(seed):
 def test_many_append_tiles_per_cta(window):
     # thousands of append tiles: every persistent CTA runs many items in a row
     rng = np.random.default_rng(700 + window)
-    B = 48
-    L = rng.integers(100, 260, size=B)
+    B = 64
+    L = rng.integers(200, 400, size=B)
     S = L + rng.integers(0, 900, size=B)
     b = W.build_batch("manytiles", 800 + window, S, L, 64, 8, layer_windows=(window,))
     run, _ = _full_check(b, what=f"manytiles w{window}")
