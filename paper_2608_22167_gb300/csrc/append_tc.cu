@@ -45,7 +45,10 @@ namespace mcpu {
 
 constexpr int kTcRows = 128;                          // rows per tile (TMEM lanes)
 constexpr int kTcKeys = 128;                          // keys per block
-constexpr int kTcKStages = 5, kTcVStages = 5;
+// Ring depths and the register cap leave room on every SM for one CTA of the
+// memory-bound decode kernel (side stream): 145 KiB of shared memory here,
+// and at most 3 warps x 144 registers on any SM sub-partition.
+constexpr int kTcKStages = 4, kTcVStages = 3;
 constexpr int kTcQBytes = kAppendTcRows * kRowBytes;  // both tiles: 32 KiB
 constexpr int kTcTileQBytes = kTcRows * kRowBytes;    // 16 KiB
 constexpr int kTcKvBytes = kTcKeys * kRowBytes;       // one K or V block: 16 KiB
@@ -138,7 +141,7 @@ __device__ __forceinline__ float chunk_exp(const uint32_t (&sv)[2][32], float sc
 
 }  // namespace
 
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __maxnreg__(144)
     append_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap qmap, const AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
