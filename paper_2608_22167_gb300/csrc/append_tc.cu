@@ -139,6 +139,32 @@ __device__ __forceinline__ float chunk_exp(const uint32_t (&sv)[2][32], float sc
   return lo_f32(ls) + hi_f32(ls);
 }
 
+// Probabilities of one chunk against the running reference m_ref (log2
+// units): p = 2^(s * scale_log2 - m_ref). The common path computes no max:
+// a chunk sum below 2^8 proves every p is below 2^8, the bound the lazy
+// rescale keeps. Otherwise (or before the first reference exists) the chunk
+// max is taken; if it exceeds m_ref by more than the threshold, m_ref is
+// raised, `alpha` is multiplied by the factor that rescales earlier
+// probabilities, and the chunk is recomputed. Returns the chunk sum.
+__device__ __forceinline__ float chunk_probs(const uint32_t (&sv)[2][32], float scale_log2, float& m_ref,
+                                             float& alpha, uint32_t (&pk)[32]) {
+  float lc = 0.f;
+  bool redo = m_ref == -INFINITY;
+  if (!redo) {
+    lc = chunk_exp(sv, scale_log2, -m_ref, pk);
+    redo = !(lc < 256.f);  // also for inf / NaN
+  }
+  if (redo) {
+    const float mx = chunk_max(sv) * scale_log2;
+    if (mx > m_ref + kRescaleThreshold) {  // also true for the first finite max
+      alpha *= ex2_approx(m_ref - mx);     // 0 when m_ref == -inf
+      m_ref = mx;
+    }
+    lc = chunk_exp(sv, scale_log2, m_ref == -INFINITY ? 0.f : -m_ref, pk);
+  }
+  return lc;
+}
+
 }  // namespace
 
 __global__ void __maxnreg__(144)
@@ -419,12 +445,7 @@ __global__ void __maxnreg__(144)
         tmem_ld_wait();
         if ((kb + 63 > wp_min) || (p.window > 0 && kb < wp_max - p.window + 1)) mask_chunk(sv, kb, pos, lo);
         float alpha = 1.f;
-        float mx = chunk_max(sv) * p.scale_log2;
-        if (mx > m_ref + kRescaleThreshold) {  // also true for the first finite max
-          alpha = ex2_approx(m_ref - mx);      // 0 when m_ref == -inf
-          m_ref = mx;
-        }
-        float l0 = chunk_exp(sv, p.scale_log2, m_ref == -INFINITY ? 0.f : -m_ref, pk);
+        float l0 = chunk_probs(sv, p.scale_log2, m_ref, alpha, pk);
         // the single P buffer was last read by PV_X(blk - 1)
         if (blk >= 1) {
           ok = __all_sync(0xffffffffu, wait_bar(bar(st.o_ready[x]), (blk - 1) & 1, abort_flag));
@@ -440,14 +461,10 @@ __global__ void __maxnreg__(144)
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(st.s_free[x]));
         if ((kb + 127 > wp_min) || (p.window > 0 && kb + 64 < wp_max - p.window + 1)) mask_chunk(sv, kb + 64, pos, lo);
-        mx = chunk_max(sv) * p.scale_log2;
-        if (__any_sync(0xffffffffu, mx > m_ref + kRescaleThreshold)) {
-          // rare: the max rose inside the block; rescale chunk 0's P too
-          float a1 = 1.f;
-          if (mx > m_ref + kRescaleThreshold) {
-            a1 = ex2_approx(m_ref - mx);
-            m_ref = mx;
-          }
+        float a1 = 1.f;
+        const float l1 = chunk_probs(sv, p.scale_log2, m_ref, a1, pk);
+        if (__any_sync(0xffffffffu, a1 != 1.f)) {
+          // rare: the reference rose inside the block; rescale chunk 0's P too
           tmem_st_wait();
           uint32_t pv[32];
           tmem_ld32(cP, pv);
@@ -461,7 +478,6 @@ __global__ void __maxnreg__(144)
           l0 *= a1;
           alpha *= a1;
         }
-        const float l1 = chunk_exp(sv, p.scale_log2, m_ref == -INFINITY ? 0.f : -m_ref, pk);
         tmem_st32(cP + 32, pk);
         l = l * alpha + (l0 + l1);
         // O_X may only be rescaled once PV_X(blk - 1) has completed (waited above)
