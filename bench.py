@@ -101,6 +101,25 @@ def peaks():
         return 6800.0, 1900.0, 1700.0, "fallback"
 
 
+# ------------------------------------------------------------------ ranks
+
+
+def max_over_ranks(values, device, world: int):
+    """Element-wise maximum of per-rank timings over all ranks (the slowest
+    rank decides); unchanged when running alone."""
+    if world <= 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], device=device, dtype=torch.float64)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return [float(x) for x in t.tolist()]
+
+
+def whole_job_gbs(bytes_per_rank: int, world: int, ms: float) -> float:
+    """Throughput of all replicas together: every rank processed its own
+    bytes_per_rank in at most `ms`."""
+    return bytes_per_rank * world / (ms * 1e-3) / 1e9
+
+
 # --------------------------------------------------------------- accounting
 
 
@@ -522,13 +541,10 @@ def run_ours(args, rank, world, dev):
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
 
     # ---- max over ranks
-    if world > 1:
-        t = torch.tensor([total_ms, e2e_ms], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms, e2e_ms = float(t[0]), float(t[1])
+    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], dev, world)
     ms_per_step = total_ms / args.steps
-    value = kv_bytes * world / (ms_per_step * 1e-3) / 1e9
-    e2e_value = kv_bytes * world / (e2e_ms * 1e-3) / 1e9
+    value = whole_job_gbs(kv_bytes, world, ms_per_step)
+    e2e_value = whole_job_gbs(kv_bytes, world, e2e_ms)
 
     res = {
         "metric": "KV-read HBM GB/s (% of GB300 peak) and attended tokens/s, paged mixed batch",
