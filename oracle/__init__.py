@@ -51,10 +51,12 @@ def _load():
             i32, i64, f64 = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
             lib.oracle_kv_append.argtypes = [P, P, P, P, P, P, P, i32, i32, i64, i32, i32, i32]
             lib.oracle_kv_append.restype = ctypes.c_int
-            lib.oracle_paged_attention.argtypes = [P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i32]
+            lib.oracle_paged_attention.argtypes = [
+                P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i32, P
+            ]
             lib.oracle_paged_attention.restype = ctypes.c_int
             lib.oracle_paged_attention_sampled.argtypes = [
-                P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i64, P, P, i32
+                P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i64, P, P, i32, P
             ]
             lib.oracle_paged_attention_sampled.restype = ctypes.c_int
             lib.oracle_double_to_bf16.argtypes = [f64]
@@ -102,9 +104,18 @@ def kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start
     return k_cache, v_cache
 
 
+def _sinks(sinks, hq):
+    if sinks is None:
+        return None, None
+    a, p = _c(sinks, np.float32)
+    assert a.shape == (hq,)
+    return a, p
+
+
 def paged_attention(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, sliding_window,
-                    softmax_scale, num_threads=0):
-    """Return (out [T, Hq, D] uint16 bf16 bits, lse [T, Hq] float32)."""
+                    softmax_scale, num_threads=0, sinks=None):
+    """Return (out [T, Hq, D] uint16 bf16 bits, lse [T, Hq] float32).
+    sinks: optional per-q-head sink logits [Hq] (natural-log units)."""
     lib = _load()
     q, q_p = _c(q, np.uint16)
     kc, kc_p = _c(k_cache, np.uint16)
@@ -115,19 +126,20 @@ def paged_attention(q, k_cache, v_cache, block_table, seq_lens, query_start_loc,
     T, hq, d = q.shape
     num_pages, hkv, page, d2 = kc.shape
     assert d == d2
+    sk, sk_p = _sinks(sinks, hq)
     out = np.zeros((T, hq, d), np.uint16)
     lse = np.zeros((T, hq), np.float32)
     rc = lib.oracle_paged_attention(
         q_p, kc_p, vc_p, bt_p, sl_p, qs_p, sl.shape[0], bt.shape[1], num_pages, hq, hkv, d, page,
         int(sliding_window), float(softmax_scale), out.ctypes.data_as(ctypes.c_void_p),
-        lse.ctypes.data_as(ctypes.c_void_p), int(num_threads),
+        lse.ctypes.data_as(ctypes.c_void_p), int(num_threads), sk_p,
     )
     _check(rc)
     return out, lse
 
 
 def paged_attention_sampled(q, k_cache, v_cache, block_table, seq_lens, query_start_loc,
-                            sliding_window, softmax_scale, tokens, heads, num_threads=0):
+                            sliding_window, softmax_scale, tokens, heads, num_threads=0, sinks=None):
     """The oracle at listed (token, q head) pairs: (out [n, D] bits, lse [n])."""
     lib = _load()
     q, q_p = _c(q, np.uint16)
@@ -141,12 +153,13 @@ def paged_attention_sampled(q, k_cache, v_cache, block_table, seq_lens, query_st
     T, hq, d = q.shape
     num_pages, hkv, page, _ = kc.shape
     n = tk.shape[0]
+    sk, sk_p = _sinks(sinks, hq)
     out = np.zeros((n, d), np.uint16)
     lse = np.zeros((n,), np.float32)
     rc = lib.oracle_paged_attention_sampled(
         q_p, kc_p, vc_p, bt_p, sl_p, qs_p, sl.shape[0], bt.shape[1], num_pages, hq, hkv, d, page,
         int(sliding_window), float(softmax_scale), tk_p, hd_p, n, out.ctypes.data_as(ctypes.c_void_p),
-        lse.ctypes.data_as(ctypes.c_void_p), int(num_threads),
+        lse.ctypes.data_as(ctypes.c_void_p), int(num_threads), sk_p,
     )
     _check(rc)
     return out, lse

@@ -38,8 +38,10 @@ def visibility(S, L, window):
 
 
 def attention(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, sliding_window,
-              softmax_scale, page_size=16):
-    """Return (out [T, Hq, D] float64, lse [T, Hq] float64), unrounded."""
+              softmax_scale, page_size=16, sinks=None):
+    """Return (out [T, Hq, D] float64, lse [T, Hq] float64), unrounded.
+    sinks: optional [Hq] logits appended to every score row as one more
+    column whose value row is zero."""
     qf = bits_to_f64(q)
     T, Hq, D = qf.shape
     Hkv = k_cache.shape[1]
@@ -59,6 +61,11 @@ def attention(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, slidi
         vq = np.repeat(v, g, axis=1)
         scores = softmax_scale * np.einsum("lhd,shd->hls", qf[t0:t1], kq)  # [Hq, L, S]
         scores = np.where(vis[None], scores, -np.inf)
+        if sinks is not None:
+            # one extra key per head: score sigma_h, value 0, always visible
+            sig = np.broadcast_to(np.asarray(sinks, np.float64)[:, None, None], (Hq, L, 1))
+            scores = np.concatenate([scores, sig], axis=2)
+            vq = np.concatenate([vq, np.zeros((1, Hq, D))], axis=0)
         m = scores.max(axis=2, keepdims=True)
         has = np.isfinite(m)
         m = np.where(has, m, 0.0)

@@ -25,6 +25,13 @@
  *         out  = sum_j exp(s_j - m) / l * V[j]          (rounded to bf16)
  *         lse  = m + ln(l)    (natural log of sum_j exp(s_j))
  *      A query with no visible key has out = 0 and lse = -inf.
+ *   3. attention sinks (optional; gpt-oss's per-head sink logits, from the
+ *      public model card, not from the paper): q head h has a logit sigma_h
+ *      that joins the normaliser but carries no value,
+ *         Z    = sum_j exp(s_j) + exp(sigma_h)
+ *         out  = sum_j exp(s_j) / Z * V[j],   lse = ln Z,
+ *      evaluated as above with m = max(max_j s_j, sigma_h). sigma_h = -inf
+ *      (or no sinks array) is step 2 exactly.
  *
  * Precision: bf16 inputs are widened exactly; every sum and product is taken
  * in double; out is rounded once, double -> bf16, to nearest-even.
@@ -35,6 +42,7 @@
  *   block_table [num_seqs, max_pages_per_seq] int32
  *   seq_lens [num_seqs] int32,  query_start_loc [num_seqs + 1] int32
  *   out [T_q, H_q, D] bf16 bits,  lse [T_q, H_q] float
+ *   sinks [H_q] float or NULL (step 3)
  *
  * Return value: 0 on success, otherwise a positive code naming the first
  * problem found (see ORACLE_ERR_*); nothing is written past a failed check.
@@ -154,13 +162,14 @@ static int64_t first_visible(int64_t p, int32_t window) {
  * pages and writes out[0..D) (bf16 bits) and *lse. */
 static int attend_one(const uint16_t* qv, const uint16_t* k_cache, const uint16_t* v_cache,
                       const int32_t* bt_row, int64_t p, int32_t kvh, int32_t window,
-                      double scale, int64_t num_pages, int32_t num_kv_heads, int32_t head_dim,
-                      int32_t page_size, double* s, double* acc, uint16_t* out, float* lse) {
+                      double scale, double sink, int64_t num_pages, int32_t num_kv_heads,
+                      int32_t head_dim, int32_t page_size, double* s, double* acc, uint16_t* out,
+                      float* lse) {
   int64_t lo = first_visible(p, window);
   int64_t n = p - lo + 1;
   if (n <= 0) {
     for (int32_t d = 0; d < head_dim; ++d) out[d] = 0;
-    *lse = -INFINITY;
+    *lse = (float)sink; /* ln exp(sigma); -inf without a sink */
     return ORACLE_OK;
   }
   /* scores */
@@ -174,9 +183,11 @@ static int attend_one(const uint16_t* qv, const uint16_t* k_cache, const uint16_
     s[j - lo] = scale * dot;
     if (s[j - lo] > m) m = s[j - lo];
   }
-  /* normaliser */
+  /* normaliser (step 3: the sink joins the max and the sum) */
+  if (sink > m) m = sink;
   double l = 0.0;
   for (int64_t j = 0; j < n; ++j) l += exp(s[j] - m);
+  if (sink > -INFINITY) l += exp(sink - m);
   /* weighted sum of values */
   for (int32_t d = 0; d < head_dim; ++d) acc[d] = 0.0;
   for (int64_t j = lo; j <= p; ++j) {
@@ -204,7 +215,7 @@ int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uin
                            int32_t max_pages_per_seq, int64_t num_pages, int32_t num_q_heads,
                            int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
                            int32_t sliding_window, double softmax_scale, uint16_t* out,
-                           float* lse, int32_t num_threads) {
+                           float* lse, int32_t num_threads, const float* sinks) {
   int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_q_heads,
                         num_kv_heads, head_dim, page_size);
   if (rc) return rc;
@@ -237,9 +248,9 @@ int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uin
         int64_t p = S - L + (t - query_start_loc[r]);
         int e = attend_one(q + (t * num_q_heads + h) * head_dim, k_cache, v_cache,
                            block_table + (int64_t)r * max_pages_per_seq, p, h / group,
-                           sliding_window, softmax_scale, num_pages, num_kv_heads, head_dim,
-                           page_size, s, acc, out + (t * num_q_heads + h) * head_dim,
-                           lse + t * num_q_heads + h);
+                           sliding_window, softmax_scale, sinks ? (double)sinks[h] : -INFINITY,
+                           num_pages, num_kv_heads, head_dim, page_size, s, acc,
+                           out + (t * num_q_heads + h) * head_dim, lse + t * num_q_heads + h);
         if (e) {
 #pragma omp atomic write
           err = e;
@@ -264,7 +275,7 @@ int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
                                    double softmax_scale, const int64_t* sample_token,
                                    const int32_t* sample_head, int64_t n_samples,
                                    uint16_t* out_samples, float* lse_samples,
-                                   int32_t num_threads) {
+                                   int32_t num_threads, const float* sinks) {
   int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_q_heads,
                         num_kv_heads, head_dim, page_size);
   if (rc) return rc;
@@ -302,8 +313,9 @@ int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
       int64_t p = S - L + (t - query_start_loc[r]);
       int e = attend_one(q + (t * num_q_heads + h) * head_dim, k_cache, v_cache,
                          block_table + (int64_t)r * max_pages_per_seq, p, h / group,
-                         sliding_window, softmax_scale, num_pages, num_kv_heads, head_dim,
-                         page_size, s, acc, out_samples + i * head_dim, lse_samples + i);
+                         sliding_window, softmax_scale, sinks ? (double)sinks[h] : -INFINITY,
+                         num_pages, num_kv_heads, head_dim, page_size, s, acc,
+                         out_samples + i * head_dim, lse_samples + i);
       if (e) {
 #pragma omp atomic write
         err = e;

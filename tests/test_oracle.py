@@ -427,3 +427,82 @@ def test_unallocated_pages_outside_the_window_are_never_read():
     assert np.any(h["block_table"] == -1)
     out, lse = _run_oracle(h)
     assert np.all(np.isfinite(lse))
+
+
+# ------------------------------------------------------- attention sinks
+
+
+def _sinks(hq, seed):
+    return np.random.default_rng(seed).normal(0.0, 1.5, size=hq).astype(np.float32)
+
+
+def test_sinks_at_minus_infinity_change_nothing():
+    b = W.fuzz_batch(21)
+    h = W.host_inputs(b)
+    out, lse = _run_oracle(h)
+    out_s, lse_s = oracle.paged_attention(h["q"], h["k_cache"], h["v_cache"], h["block_table"], h["seq_lens"],
+                                          h["query_start_loc"], h["sliding_window"], h["softmax_scale"],
+                                          sinks=np.full(b.num_q_heads, -np.inf, np.float32))
+    assert np.array_equal(out, out_s) and np.array_equal(lse, lse_s)
+
+
+@pytest.mark.parametrize("sigma,frac", [(0.0, 0.5), (math.log(3.0), 0.25), (-math.log(3.0), 0.75)])
+def test_sink_with_one_visible_key_closed_form(sigma, frac):
+    # q = 0 and window 1: one key with score 0; the sink adds e^sigma to the
+    # normaliser, so out = v / (1 + e^sigma) and lse = ln(1 + e^sigma).
+    b = W.build_batch("sink1", 31, [9, 40], [1, 3], 4, 2, layer_windows=(1,))
+    h = W.host_inputs(b)
+    h["q"] = np.zeros_like(h["q"])
+    kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                              h["seq_lens"], h["query_start_loc"])
+    out, lse = oracle.paged_attention(h["q"], kc, vc, h["block_table"], h["seq_lens"], h["query_start_loc"], 1,
+                                      h["softmax_scale"], sinks=np.full(4, sigma, np.float32))
+    vals = brute.bits_to_f64(h["v_new"])  # the query's own key is its new row
+    for t in range(out.shape[0]):
+        for hq in range(4):
+            want = vals[t, hq // 2] * frac
+            assert np.all(np.abs(_f(out[t, hq]) - want) <= np.abs(want) * 2.0**-8)
+            assert abs(lse[t, hq] - math.log1p(math.exp(np.float32(sigma)))) <= 1e-6
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_sinks_match_brute_force(seed):
+    b = W.fuzz_batch(300 + seed)
+    h = W.host_inputs(b)
+    kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                              h["seq_lens"], h["query_start_loc"])
+    sk = _sinks(b.num_q_heads, seed)
+    out, lse = oracle.paged_attention(h["q"], kc, vc, h["block_table"], h["seq_lens"], h["query_start_loc"],
+                                      h["sliding_window"], h["softmax_scale"], sinks=sk)
+    ref_out, ref_lse = brute.attention(h["q"], kc, vc, h["block_table"], h["seq_lens"], h["query_start_loc"],
+                                       h["sliding_window"], h["softmax_scale"], sinks=sk)
+    _assert_close_to_exact(out, lse, ref_out, ref_lse)
+
+
+def test_sink_rescales_the_sinkless_result():
+    # Z' = Z + e^sigma: lse' = logaddexp(lse, sigma) and out' = out * e^(lse - lse')
+    b = W.fuzz_batch(44)
+    h = W.host_inputs(b)
+    sk = _sinks(b.num_q_heads, 7)
+    out, lse = _run_oracle(h)
+    out_s, lse_s = oracle.paged_attention(h["q"], h["k_cache"], h["v_cache"], h["block_table"], h["seq_lens"],
+                                          h["query_start_loc"], h["sliding_window"], h["softmax_scale"], sinks=sk)
+    want_lse = np.logaddexp(lse.astype(np.float64), sk[None, :].astype(np.float64))
+    assert np.allclose(lse_s, want_lse, rtol=0, atol=2e-6 * np.maximum(1, np.abs(want_lse)).max())
+    want = _f(out) * np.exp(lse.astype(np.float64) - want_lse)[..., None]
+    assert np.all(np.abs(_f(out_s) - want) <= np.abs(want) * 2.0**-7 + 1e-30)
+
+
+def test_sampled_evaluation_with_sinks_equals_full_evaluation():
+    b = W.fuzz_batch(45)
+    h = W.host_inputs(b)
+    sk = _sinks(b.num_q_heads, 9)
+    out, lse = oracle.paged_attention(h["q"], h["k_cache"], h["v_cache"], h["block_table"], h["seq_lens"],
+                                      h["query_start_loc"], h["sliding_window"], h["softmax_scale"], sinks=sk)
+    rng = np.random.default_rng(3)
+    toks = rng.integers(0, out.shape[0], size=20).astype(np.int64)
+    heads = rng.integers(0, b.num_q_heads, size=20).astype(np.int32)
+    so, sl = oracle.paged_attention_sampled(h["q"], h["k_cache"], h["v_cache"], h["block_table"], h["seq_lens"],
+                                            h["query_start_loc"], h["sliding_window"], h["softmax_scale"], toks,
+                                            heads, sinks=sk)
+    assert np.array_equal(so, out[toks, heads]) and np.array_equal(sl, lse[toks, heads])
