@@ -106,6 +106,12 @@ typedef struct mcpu_options {
    * Under stream capture they become event-record nodes of the graph, so
    * every replay records them. */
   void* const* phase_events;
+  /* Optional attention sinks (gpt-oss; not in the paper): device pointer to
+   * H_q floats, the sink logit sigma_h of each q head in natural-log units,
+   * or NULL. A sink joins the softmax normaliser and carries no value:
+   * out = sum_j e^{s_j} V_j / (sum_j e^{s_j} + e^{sigma_h}) and lse is the
+   * log of that normaliser. 4-byte aligned; read by the kernels only. */
+  const float* sinks;
 } mcpu_options;
 #define MCPU_NUM_PHASE_EVENTS 6
 

@@ -149,7 +149,7 @@ mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : cuda_
 
 extern "C" {
 
-int32_t mcpu_abi_version(void) { return 1; }
+int32_t mcpu_abi_version(void) { return 2; }
 
 int32_t mcpu_last_cuda_error(void) { return t_last_cuda_error; }
 
@@ -213,6 +213,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
     return MCPU_ERR_INVALID_ARG;
   if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
   if (opts && opts->split_pages < 0) return MCPU_ERR_INVALID_ARG;
+  if (opts && opts->sinks && !aligned(opts->sinks, 4)) return MCPU_ERR_INVALID_ARG;
 
   DeviceState* dev = nullptr;
   st = device_state(&dev);
@@ -248,6 +249,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   p.cascade_enabled = (opts && (opts->flags & MCPU_FLAG_NO_CASCADE)) ? 0 : 1;
   p.oob_row = (int32_t)rows;
   p.append_tile_tok = (legacy_append ? kAppendRowsMin : kAppendTcRows) / p.group;
+  p.sinks = opts ? opts->sinks : nullptr;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   void* const* ev = opts ? opts->phase_events : nullptr;

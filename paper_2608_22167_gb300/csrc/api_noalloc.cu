@@ -172,6 +172,7 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
   p.cascade_enabled = 0;
   p.oob_row = (int32_t)rows;
   p.append_tile_tok = kAppendTcRows / group;
+  p.sinks = nullptr;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // The scratch keeps the previous call's contents: the status word must

@@ -230,7 +230,12 @@ __global__ void __launch_bounds__(kAppWarps * 32)
       l0 += __shfl_xor_sync(0xffffffffu, l0, off);
       l1 += __shfl_xor_sync(0xffffffffu, l1, off);
     }
-    const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f, inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
+    float inv0 = l0 > 0.f ? 1.f / l0 : 0.f, inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
+    float b0 = l0 > 0.f ? m0 + __log2f(l0) : -INFINITY, b1 = l1 > 0.f ? m1 + __log2f(l1) : -INFINITY;
+    if (p.sinks != nullptr) {  // the sink joins the normaliser
+      inv0 = finish_with_sink(m0, l0, sink_log2(p, kvh * g + r0 % g), &b0);
+      inv1 = finish_with_sink(m1, l1, sink_log2(p, kvh * g + r1 % g), &b1);
+    }
     const size_t orow0 = ((size_t)(a.token_begin + tk0) * Hq + kvh * g + r0 % g);
     const size_t orow1 = ((size_t)(a.token_begin + tk1) * Hq + kvh * g + r1 % g);
 #pragma unroll
@@ -242,8 +247,8 @@ __global__ void __launch_bounds__(kAppWarps * 32)
         *reinterpret_cast<uint32_t*>(p.out + orow1 * kHeadDim + d) = pack_bf16x2(o[nt][2] * inv1, o[nt][3] * inv1);
     }
     if ((lane & 3) == 0) {
-      if (ok0) p.lse[orow0] = l0 > 0.f ? (m0 + __log2f(l0)) * 0.69314718055994531f : -INFINITY;
-      if (ok1) p.lse[orow1] = l1 > 0.f ? (m1 + __log2f(l1)) * 0.69314718055994531f : -INFINITY;
+      if (ok0) p.lse[orow0] = b0 * 0.69314718055994531f;
+      if (ok1) p.lse[orow1] = b1 * 0.69314718055994531f;
     }
   }
 }

@@ -515,7 +515,9 @@ __global__ void __maxnreg__(144)
         mbar_arrive(bar(st.item_empty[slot]));
       }
       if (valid) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
+        float inv = l > 0.f ? 1.f / l : 0.f;
+        float lse2 = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
+        if (p.sinks != nullptr) inv = finish_with_sink(m_ref, l, sink_log2(p, kvh * g + head), &lse2);
         const size_t orow = (size_t)(a.token_begin + tok) * Hq + kvh * g + head;
         uint4* dst = reinterpret_cast<uint4*>(p.out + orow * kHeadDim);
 #pragma unroll
@@ -528,7 +530,7 @@ __global__ void __maxnreg__(144)
           w.w = pack_bf16x2(__uint_as_float(ov[h][e0 + 6]) * inv, __uint_as_float(ov[h][e0 + 7]) * inv);
           dst[v] = w;
         }
-        p.lse[orow] = l > 0.f ? (m_ref + __log2f(l)) * 0.69314718055994531f : -INFINITY;
+        p.lse[orow] = lse2 * 0.69314718055994531f;
       }
     }
   }

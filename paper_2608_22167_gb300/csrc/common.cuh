@@ -122,7 +122,29 @@ struct AttnParams {
   int32_t cascade_enabled;
   int32_t oob_row;               // y coordinate just past the pool, read as zeros
   int32_t append_tile_tok;       // tokens per append tile (tile rows / group)
+  const float* sinks;            // [Hq] sink logits (natural log), or null
 };
+
+// Attention sinks (gpt-oss): q head h has a logit sigma_h that joins the
+// softmax normaliser and carries no value. sink_log2 is sigma_h in base-2
+// units (-inf without sinks). finish_with_sink normalises an accumulator held
+// relative to the base-2 running max m with row sum l, the sink included:
+// returns the factor the accumulator is multiplied by and writes the base-2
+// log normaliser; m may be -inf (no visible key).
+__device__ __forceinline__ float sink_log2(const AttnParams& p, int h) {
+  return p.sinks ? p.sinks[h] * 1.4426950408889634f : -INFINITY;
+}
+__device__ __forceinline__ float finish_with_sink(float m, float l, float s2, float* lse2) {
+  const float M = fmaxf(m, s2);
+  if (!(M > -INFINITY)) {
+    *lse2 = -INFINITY;
+    return 0.f;
+  }
+  const float a = m > -INFINITY ? exp2f(m - M) : 0.f;
+  const float lt = l * a + (s2 > -INFINITY ? exp2f(s2 - M) : 0.f);
+  *lse2 = M + __log2f(lt);
+  return a / lt;
+}
 
 __device__ __forceinline__ PlanHeader* header(const AttnParams& p) {
   return reinterpret_cast<PlanHeader*>(p.ws + p.lay.header);

@@ -265,13 +265,17 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
       for (int e = 0; e < 2; ++e) {
         const int qv = nt * 8 + 2 * (lane & 3) + e;
         const float l = l_run[nt][e];
-        const float inv = l > 0.f ? 1.f / l : 0.f;
+        float inv = l > 0.f ? 1.f / l : 0.f;
+        float lse2 = l > 0.f ? m_run[nt][e] + __log2f(l) : -INFINITY;
+        // a row finished here (one split) takes its sink now; split rows in the merge
+        if (NT == 1 && p.sinks != nullptr && slot < 0 && qv < g)
+          inv = finish_with_sink(m_run[nt][e], l, sink_log2(p, kvh * g + qv), &lse2);
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
           so[qv * kLd + mt * 16 + (lane >> 2)] = acc[mt][nt][e] * inv;
           so[qv * kLd + mt * 16 + (lane >> 2) + 8] = acc[mt][nt][e + 2] * inv;
         }
-        if ((lane >> 2) == 0) sl[qv] = l > 0.f ? m_run[nt][e] + __log2f(l) : -INFINITY;
+        if ((lane >> 2) == 0) sl[qv] = lse2;
       }
     }
     __syncwarp();

@@ -4,7 +4,8 @@
 // for GRPO-group members the shared-prefix part) has, per query head, parts
 // i with a normalised output o_i and a base-2 log normaliser b_i. Exactly:
 //   b = b_max + log2(sum_i 2^(b_i - b_max)),  out = sum_i 2^(b_i - b) o_i,
-// and the reported lse is b * ln 2. One warp merges one (row, head); each
+// and the reported lse is b * ln 2. An attention sink sigma adds a part
+// 2^(sigma log2 e) with no value. One warp merges one (row, head); each
 // lane owns two of the 64 dims.
 #include "common.cuh"
 
@@ -25,7 +26,10 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
     const int h = w % Hq;
     float bmax = -INFINITY;
     for (int i = 0; i < mr.n_parts; ++i) bmax = fmaxf(bmax, lse_part[(size_t)(mr.part_off + i) * Hq + h]);
-    float sum = 0.f, o0 = 0.f, o1 = 0.f;
+    // an attention sink joins the normaliser as one more part with no value
+    const float s2 = sink_log2(p, h);
+    bmax = fmaxf(bmax, s2);
+    float sum = s2 > -INFINITY ? fast_exp2(s2 - bmax) : 0.f, o0 = 0.f, o1 = 0.f;
     if (bmax != -INFINITY) {
       for (int i = 0; i < mr.n_parts; ++i) {
         const size_t idx = (size_t)(mr.part_off + i) * Hq + h;

@@ -69,7 +69,8 @@ class Dims(ctypes.Structure):
 
 
 class Options(ctypes.Structure):
-    _fields_ = [("flags", ctypes.c_uint32), ("split_pages", ctypes.c_int32), ("phase_events", ctypes.c_void_p)]
+    _fields_ = [("flags", ctypes.c_uint32), ("split_pages", ctypes.c_int32), ("phase_events", ctypes.c_void_p),
+                ("sinks", ctypes.c_void_p)]
 
 
 NUM_PHASE_EVENTS = 6
@@ -170,11 +171,16 @@ def mcpu_kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_
 
 def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, sliding_window,
                                  softmax_scale, out, lse, workspace, flags=0, split_pages=0, stream=None,
-                                 phase_events=None):
+                                 phase_events=None, sinks=None):
     """phase_events: optional list of NUM_PHASE_EVENTS torch.cuda.Event the
-    call records around its kernels (see mcpu_options in include/mcpu.h)."""
+    call records around its kernels (see mcpu_options in include/mcpu.h);
+    sinks: optional float32 device tensor [H_q] of attention-sink logits."""
     d = dims(q, k_cache, block_table, seq_lens)
-    opts = Options(flags=int(flags), split_pages=int(split_pages), phase_events=None)
+    opts = Options(flags=int(flags), split_pages=int(split_pages), phase_events=None, sinks=None)
+    if sinks is not None:
+        if sinks.dtype != torch.float32 or sinks.numel() != d.num_q_heads or not sinks.is_cuda:
+            raise ValueError("sinks must be a float32 CUDA tensor with one value per q head")
+        opts.sinks = ctypes.c_void_p(sinks.data_ptr())
     if phase_events is not None:
         assert len(phase_events) == NUM_PHASE_EVENTS
         if any(e.cuda_event == 0 for e in phase_events):

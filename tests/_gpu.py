@@ -50,10 +50,12 @@ class Run:
         mcpu.mcpu_kv_append(self.k_new, self.v_new, self.kc, self.vc, self.bt, self.sl, self.qsl,
                             mcpu.status_word(self.ws))
 
-    def forward(self, flags=0, split_pages=0):
+    def forward(self, flags=0, split_pages=0, sinks=None):
+        """sinks: optional numpy float32 [H_q] attention-sink logits."""
+        sk = None if sinks is None else torch.from_numpy(np.asarray(sinks, np.float32)).to(self.q.device)
         mcpu.mcpu_paged_attention_forward(self.q, self.kc, self.vc, self.bt, self.sl, self.qsl, self.window,
                                           self.batch.softmax_scale, self.out, self.lse, self.ws, flags=flags,
-                                          split_pages=split_pages)
+                                          split_pages=split_pages, sinks=sk)
 
     def status(self):
         return mcpu.mcpu_read_device_status(self.ws)
@@ -67,17 +69,17 @@ class Run:
         return self.out.float().cpu().numpy(), self.lse.cpu().numpy()
 
 
-def oracle_full(batch: W.Batch, layer: int = 0):
+def oracle_full(batch: W.Batch, layer: int = 0, sinks=None):
     """Oracle outputs of a whole (small) layer, append applied first."""
     h = W.host_inputs(batch, layer)
     kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
                               h["seq_lens"], h["query_start_loc"])
     out, lse = oracle.paged_attention(h["q"], kc, vc, h["block_table"], h["seq_lens"], h["query_start_loc"],
-                                      h["sliding_window"], h["softmax_scale"])
+                                      h["sliding_window"], h["softmax_scale"], sinks=sinks)
     return oracle.bf16_bits_to_float(out), lse, (kc, vc)
 
 
-def oracle_sampled(batch: W.Batch, rows, n_per_row: int, rng, layer: int = 0):
+def oracle_sampled(batch: W.Batch, rows, n_per_row: int, rng, layer: int = 0, sinks=None):
     """Oracle at sampled (token, head) pairs of the given rows: returns
     (token indices in the batch, heads, out [n, D], lse [n])."""
     h = W.host_rows(batch, rows, layer)
@@ -97,7 +99,7 @@ def oracle_sampled(batch: W.Batch, rows, n_per_row: int, rng, layer: int = 0):
     toks = np.asarray(toks, np.int64)
     heads = np.asarray(heads, np.int32)
     out, lse = oracle.paged_attention_sampled(h["q"], kc, vc, h["block_table"], h["seq_lens"], qsl,
-                                              h["sliding_window"], h["softmax_scale"], toks, heads)
+                                              h["sliding_window"], h["softmax_scale"], toks, heads, sinks=sinks)
     return h["token_map"][toks], heads, oracle.bf16_bits_to_float(out), lse
 
 

@@ -14,13 +14,13 @@ if torch.cuda.is_available():
     from paper_2608_22167_gb300 import mcpu
 
 
-def _full_check(batch, layer=0, flags=0, split_pages=0, what=""):
+def _full_check(batch, layer=0, flags=0, split_pages=0, what="", sinks=None):
     run = Run(batch, layer)
     run.append()
-    run.forward(flags=flags, split_pages=split_pages)
+    run.forward(flags=flags, split_pages=split_pages, sinks=sinks)
     code, bits = run.status()
     assert code == 0, f"device status bits {bits}"
-    ref_out, ref_lse, (okc, ovc) = oracle_full(batch, layer)
+    ref_out, ref_lse, (okc, ovc) = oracle_full(batch, layer, sinks=sinks)
     assert np.array_equal(W.to_host(run.kc), okc), "k pool differs after append"
     assert np.array_equal(W.to_host(run.vc), ovc), "v pool differs after append"
     got_out, got_lse = run.out_host()
@@ -278,3 +278,66 @@ def test_cuda_graph_replay_follows_new_lengths():
     got_out, got_lse = run.out_host()
     assert_parity(got_out, got_lse, ref_out, ref_lse, "graph replay, new lengths")
     assert np.abs(got_out - out_e).max() > 0  # the replay did compute the new batch
+
+
+# ------------------------------------------------------- attention sinks
+
+
+def _sinks(hq, seed):
+    return np.random.default_rng(seed).normal(0.0, 1.5, size=hq).astype(np.float32)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_sinks_fuzz(seed):
+    b = W.fuzz_batch(900 + seed, max_len=2000, max_chunk=200)
+    _full_check(b, what=f"sinks fuzz{seed}", sinks=_sinks(b.num_q_heads, seed))
+
+
+@pytest.mark.parametrize("split_pages", [1, 3])
+def test_sinks_on_split_rows(split_pages):
+    # split rows take their sink in the merge, unsplit rows in the decode kernel
+    b = W.build_batch("sinksplit", 56, [700, 33, 2049, 16, 1], [1, 1, 1, 1, 1], 32, 8)
+    run, _ = _full_check(b, split_pages=split_pages, what=f"sinks split{split_pages}", sinks=_sinks(32, 1))
+    assert run.header()["n_merge"] > 0
+
+
+def test_sinks_with_cascade_groups():
+    b = _grouped_batch(4)
+    run, _ = _full_check(b, what="sinks cascade", sinks=_sinks(64, 2))
+    assert run.header()["n_cascade"] > 0
+
+
+@pytest.mark.parametrize("window", [16, 128])
+def test_sinks_with_windows(window):
+    rng = np.random.default_rng(window + 5)
+    S = rng.integers(1, 2500, size=6)
+    L = np.where(np.arange(6) % 2 == 0, 1, np.minimum(S, rng.integers(2, 300, size=6)))
+    b = W.build_batch("sinkwin", 78 + window, S, L, 64, 8, layer_windows=(window,))
+    _full_check(b, what=f"sinks window{window}", sinks=_sinks(64, 3))
+
+
+def test_sinks_on_both_append_kernels():
+    rng = np.random.default_rng(57)
+    S = rng.integers(200, 3000, size=4)
+    L = np.minimum(S, rng.integers(2, 400, size=4))
+    b = W.build_batch("sinkapp", 58, S, L, 16, 2)
+    sk = _sinks(16, 4)
+    _full_check(b, what="sinks tcgen05 append", sinks=sk)
+    _full_check(b, flags=mcpu.FLAG_MMA_SYNC_APPEND, what="sinks mma.sync append", sinks=sk)
+
+
+def test_sinks_mixed_batch_sampled():
+    b = W.config_mixed(device="cuda")
+    sk = _sinks(b.num_q_heads, 5)
+    run = Run(b)
+    run.append()
+    run.forward(sinks=sk)
+    assert run.status()[0] == 0
+    L = b.q_lens
+    app = list(np.nonzero(L > 1)[0])
+    dec = list(np.nonzero(L == 1)[0])
+    rows = sorted(app[:4] + dec[:6])
+    rng = np.random.default_rng(12)
+    toks, heads, ref_out, ref_lse = oracle_sampled(b, rows, 16, rng, sinks=sk)
+    got_out, got_lse = run.out_host()
+    assert_parity(got_out[toks, heads], got_lse[toks, heads], ref_out, ref_lse, "mixed with sinks")
