@@ -593,6 +593,135 @@ def run_ours(args, rank, world, dev):
     return res
 
 
+CHURN_DESC = ("rollout simulator: 48 GRPO groups x 8 live trajectories, prompts U[1024,8192] shared per group, "
+              "responses logU[16,256] tokens per turn, tool waits U[2,20] steps, observations logU[64,1024], "
+              "2-6 turns, max 32768 tokens; 64q/8kv, D=64, page 16, bf16; the batch changes every step")
+
+
+def churn_config():
+    from paper_2608_22167_gb300.rollout_sim import SimConfig
+
+    return SimConfig(num_pages=1 << 20, max_pages_per_seq=2048, max_live_groups=48, group_size=8,
+                     prompt_len=(1024, 8192), response_len=(16, 256), observation_len=(64, 1024),
+                     tool_wait_steps=(2, 20), acquire_steps=(0, 4), max_turns=(2, 6), max_len=32768)
+
+
+def run_churn(args, rank, world, dev):
+    """The path fed by the rollout simulator: every step the batch changes
+    (trajectories join after acquiring an environment, decode, stop on tool
+    calls, append observations, finish). The simulator first runs
+    `--churn-settle` host-only steps so the timed steps see a settled mix of
+    lengths and states; the KV pool is filled with N(0,1) values once."""
+    from paper_2608_22167_gb300 import mcpu
+    from paper_2608_22167_gb300.rollout_sim import RolloutSim
+
+    hbm, tc_burst, _, peak_src = peaks()
+    cfg = churn_config()
+    sim = RolloutSim(cfg, seed=2001 + 7 * rank)
+    Hq, Hkv, D = 64, 8, 64
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(2002 + rank)
+    kc = torch.randn((cfg.num_pages, Hkv, 16, D), generator=gen, device=dev, dtype=torch.bfloat16)
+    vc = torch.randn((cfg.num_pages, Hkv, 16, D), generator=gen, device=dev, dtype=torch.bfloat16)
+    max_t = 1 << 16  # query tokens of one step (a prefill of 8192 plus decodes and observations)
+    qbuf = torch.randn((max_t, Hq, D), generator=gen, device=dev, dtype=torch.bfloat16)
+    knbuf = torch.randn((max_t, Hkv, D), generator=gen, device=dev, dtype=torch.bfloat16)
+    vnbuf = torch.randn((max_t, Hkv, D), generator=gen, device=dev, dtype=torch.bfloat16)
+    out = torch.empty_like(qbuf)
+    lse = torch.empty((max_t, Hq), dtype=torch.float32, device=dev)
+    for _ in range(args.churn_settle):
+        sim.step()
+    stream = torch.cuda.current_stream()
+
+    def one_step(record):
+        b = sim.step()
+        if b.num_seqs == 0:
+            return None
+        T = b.total_q
+        if T > max_t:
+            raise RuntimeError(f"a step with {T} query tokens exceeds the bench's buffers")
+        bt = torch.from_numpy(b.block_table).to(dev)
+        sl = torch.from_numpy(b.seq_lens).to(dev)
+        qsl = torch.from_numpy(b.query_start_loc).to(dev)
+        q, kn, vn = qbuf[:T], knbuf[:T], vnbuf[:T]
+        d = mcpu.dims(q, kc, bt, sl)
+        ws = mcpu.new_workspace(d, dev)
+        e0 = e1 = None
+        if record:
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        mcpu.mcpu_kv_append(kn, vn, kc, vc, bt, sl, qsl, mcpu.status_word(ws))
+        mcpu.mcpu_paged_attention_forward(q, kc, vc, bt, sl, qsl, 0, 0.125, out[:T], lse[:T], ws)
+        if record:
+            e1.record(stream)
+        # KV bytes: every visible token once, shared prompt pages once per group
+        S = b.seq_lens.astype(np.int64)
+        kv_tokens = int(S.sum())
+        for g in np.unique(b.groups):
+            rows = np.nonzero(b.groups == g)[0]
+            if len(rows) < 2:
+                continue
+            ref = b.block_table[rows[0]]
+            lim = int(S[rows].min() // 16)
+            n = 0
+            while n < lim and np.all(b.block_table[rows, n] == ref[n]):
+                n += 1
+            kv_tokens -= (len(rows) - 1) * n * 16
+        L = b.q_lens.astype(np.int64)
+        pairs = int((L * (S - L) + L * (L + 1) // 2).sum())  # query i sees S - L + i + 1 keys
+        return dict(ws=ws, ev=(e0, e1), kv_bytes=kv_tokens * 2 * Hkv * D * 2, rows=b.num_seqs, T=T,
+                    append_rows=int((L > 1).sum()), pairs=pairs)
+
+    for _ in range(args.warmup):
+        one_step(False)
+    torch.cuda.synchronize()
+    recs = []
+    wall0 = time.perf_counter()
+    for _ in range(args.steps):
+        r = one_step(True)
+        if r is not None:
+            recs.append(r)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    for r in recs:
+        code, bits = mcpu.mcpu_read_device_status(r["ws"])
+        if code != 0:
+            raise RuntimeError(f"device status {bits}")
+    dev_ms = [r["ev"][0].elapsed_time(r["ev"][1]) for r in recs]
+    tot_ms = float(sum(dev_ms))
+    kv = sum(r["kv_bytes"] for r in recs)
+    tot_ms_all = max_over_ranks([tot_ms], dev, world)[0]
+    value = whole_job_gbs(kv // max(world, 1), world, tot_ms_all) if world > 1 else kv / (tot_ms * 1e-3) / 1e9
+    return {
+        "metric": "KV-read HBM GB/s (% of GB300 peak) and attended tokens/s, paged mixed batch",
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": len(recs),
+        "warmup": args.warmup,
+        "ms_per_step": round(tot_ms_all / max(len(recs), 1), 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V; the batch sequence drawn by the rollout simulator)",
+        "config": {"workload": CHURN_DESC, "layers": 1, "settle_steps": args.churn_settle,
+                   "mean_rows": round(float(np.mean([r["rows"] for r in recs])), 1),
+                   "mean_query_tokens": round(float(np.mean([r["T"] for r in recs])), 1),
+                   "mean_append_rows": round(float(np.mean([r["append_rows"] for r in recs])), 2),
+                   "l2": "KV pool 34 GB >> 126 MB L2; no flush",
+                   "parallelism": f"replicas x{world} (no exchange step)",
+                   "launch": "eager; device time per step from CUDA events around the C-ABI calls"},
+        "frac_of_hbm_peak": round(value / max(world, 1) / hbm, 4),
+        "attended_tokens_per_s": round(sum(r["pairs"] for r in recs) / (tot_ms * 1e-3), 1),
+        "generated_tokens_per_s": round(sum(r["T"] for r in recs) / (tot_ms * 1e-3), 1),
+        "gpu_launches": 6 * len(recs),
+        "wall_s_timed": round(wall, 3),
+        "peak_source": peak_src,
+    }
+
+
 def run_reference(args, rank, world):
     """The oracle (plain CPU definition) timed on the host cores, rank 0 only."""
     if rank != 0:
@@ -637,7 +766,9 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(W.CONFIGS), default="mixed")
+    ap.add_argument("--workload", choices=sorted(W.CONFIGS) + ["churn"], default="mixed")
+    ap.add_argument("--churn-settle", type=int, default=400,
+                    help="host-only simulator steps before the churn workload's first GPU step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--launch", choices=["graph", "eager"], default="eager",
@@ -665,7 +796,7 @@ def main():
         from __graft_entry__ import build
 
         build()
-        res = run_ours(args, rank, world, dev)
+        res = run_churn(args, rank, world, dev) if args.workload == "churn" else run_ours(args, rank, world, dev)
     if rank == 0 and res is not None:
         print(json.dumps(res))
     if world > 1:
