@@ -341,3 +341,67 @@ def test_sinks_mixed_batch_sampled():
     toks, heads, ref_out, ref_lse = oracle_sampled(b, rows, 16, rng, sinks=sk)
     got_out, got_lse = run.out_host()
     assert_parity(got_out[toks, heads], got_lse[toks, heads], ref_out, ref_lse, "mixed with sinks")
+
+
+# ------------------------------------------------- bad inputs and limits
+
+
+def _good_rows_parity(run, b, good, what):
+    rng = np.random.default_rng(77)
+    toks, heads, ref_out, ref_lse = oracle_sampled(b, good, 24, rng)
+    got_out, got_lse = run.out_host()
+    assert_parity(got_out[toks, heads], got_lse[toks, heads], ref_out, ref_lse, what)
+
+
+def test_bad_page_ids_are_reported_and_other_rows_are_unaffected():
+    # pages outside the pool (too large, negative) in a decode row and in an
+    # append row: the kernels check every page id, load zeros instead and
+    # raise MCPU_ERR_BAD_PAGE; rows with valid tables are computed as usual
+    S = [900, 300, 1200, 77, 500, 260]
+    L = [1, 40, 1, 1, 90, 1]
+    b = W.build_batch("badpage", 71, S, L, 16, 2)
+    run = Run(b)
+    n_pages = run.kc.shape[0]
+    run.bt[0, 3] = n_pages + 3
+    run.bt[1, 10] = -7
+    run.append()
+    run.forward()
+    code, bits = run.status()
+    assert code == 5, (code, bits)  # MCPU_ERR_BAD_PAGE
+    assert bits & mcpu.STATUS_BAD_PAGE
+    _good_rows_parity(run, b, [2, 3, 4, 5], "rows next to bad pages")
+
+
+def test_inconsistent_lengths_are_reported():
+    S = [400, 300, 700, 50]
+    L = [1, 30, 1, 1]
+    b = W.build_batch("badlen", 72, S, L, 16, 2)
+    run = Run(b)
+    run.sl[1] = 10  # L = 30 > S = 10: the row is skipped
+    run.append()
+    run.forward()
+    code, bits = run.status()
+    assert code == 6 and bits & mcpu.STATUS_BAD_LENGTHS, (code, bits)  # MCPU_ERR_BAD_LENGTHS
+    _good_rows_parity(run, b, [0, 2, 3], "rows next to a bad length")
+    # query_start_loc that does not end at total_q: nothing is planned
+    run2 = Run(b)
+    run2.qsl[-1] = int(b.total_q) - 1
+    run2.forward()
+    code, bits = run2.status()
+    assert code == 6 and bits & mcpu.STATUS_BAD_LENGTHS
+    assert run2.header()["n_decode"] == 0 and run2.header()["n_append"] == 0
+
+
+def test_largest_row_count():
+    # 2048 rows (the planner's limit), short decode and append rows mixed
+    rng = np.random.default_rng(73)
+    B = 2048
+    S = rng.integers(1, 400, size=B)
+    L = np.where(rng.random(B) < 0.05, np.minimum(S, rng.integers(2, 40, size=B)), 1)
+    b = W.build_batch("rows2048", 74, S, L, 16, 2)
+    run = Run(b)
+    run.append()
+    run.forward()
+    assert run.status()[0] == 0
+    rows = sorted(rng.choice(B, size=40, replace=False))
+    _good_rows_parity(run, b, rows, "2048 rows")
