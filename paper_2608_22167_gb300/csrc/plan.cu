@@ -19,16 +19,19 @@ namespace mcpu {
 
 namespace {
 
-constexpr int kWarps = kPlanThreads / 32;
+// The planner runs as one CTA of NT threads (256 for up to 512 rows, else
+// 1024), each owning R = 2 consecutive rows for the scans.
 constexpr int R = kRowsPerPlanThread;  // rows owned by each thread: tid * R + i
 
 struct ScanBuf {
-  int warp[kWarps + 1];
+  int warp[kPlanThreads / 32 + 1];
 };
 
 // Exclusive prefix sum over the whole CTA of one value per thread; the CTA
 // total is returned through *total. Every thread must call it.
+template <int NT>
 __device__ int cta_scan(int v, int* total, ScanBuf& sb) {
+  constexpr int kWarps = NT / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int x = v;
 #pragma unroll
@@ -39,15 +42,15 @@ __device__ int cta_scan(int v, int* total, ScanBuf& sb) {
   if (lane == 31) sb.warp[warp] = x;
   __syncthreads();
   if (warp == 0) {
-    int s = sb.warp[lane];
+    const int s = lane < kWarps ? sb.warp[lane] : 0;
     int t = s;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       int y = __shfl_up_sync(0xffffffffu, t, o);
       if (lane >= o) t += y;
     }
-    sb.warp[lane] = t - s;
-    if (lane == 31) sb.warp[kWarps] = t;
+    if (lane < kWarps) sb.warp[lane] = t - s;
+    if (lane == kWarps - 1) sb.warp[kWarps] = t;
   }
   __syncthreads();
   const int res = sb.warp[warp] + x - v;
@@ -58,6 +61,7 @@ __device__ int cta_scan(int v, int* total, ScanBuf& sb) {
 
 // Exclusive scan of a per-row array in shared memory (rows tid*R .. +R-1),
 // written back in place; returns the total.
+template <int NT>
 __device__ int scan_rows(int* a, int B, ScanBuf& sb) {
   int v[R], s = 0;
 #pragma unroll
@@ -67,7 +71,7 @@ __device__ int scan_rows(int* a, int B, ScanBuf& sb) {
     s += v[i];
   }
   int total;
-  int base = cta_scan(s, &total, sb);
+  int base = cta_scan<NT>(s, &total, sb);
 #pragma unroll
   for (int i = 0; i < R; ++i) {
     const int r = threadIdx.x * R + i;
@@ -123,7 +127,9 @@ struct PlanSmem {
   int split_pages;
 };
 
-__global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
+template <int NT>
+__global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
+  constexpr int kWarps = NT / 32;
   extern __shared__ __align__(16) uint8_t plan_smem_raw[];
   PlanSmem& sm = *reinterpret_cast<PlanSmem*>(plan_smem_raw);
   PlanHeader* hdr = header(p);
@@ -148,7 +154,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   }
 
   // ---- phase 1: per-row kind and lengths
-  for (int r = tid; r < B; r += kPlanThreads) {
+  for (int r = tid; r < B; r += NT) {
     const int q0 = p.qsl[r], q1 = p.qsl[r + 1];
     const int len = q1 - q0, s = p.seq_lens[r];
     const bool bad = len < 0 || s < len || s > p.max_pages * kPage;
@@ -166,17 +172,46 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   __syncthreads();
 
   // ---- phase 2: shared-prefix groups (full-context calls only)
+  // lcp[r] = leading physical pages row r shares with row r - 1 (full pages
+  // of both). First the leading kLcpProbe pages of every adjacent pair are
+  // compared by all threads at once (most pairs differ at once, group
+  // members agree over the probe); pairs that agree over the whole probe go
+  // on warp by warp, 128 entries per step.
+  constexpr int kLcpProbe = 32;
   const bool cascade = p.cascade_enabled && p.window <= 0;
   if (cascade) {
+    for (int r = tid; r < B; r += NT) {
+      const int sa = r > 0 ? sm.S[r - 1] : -1, sb = sm.S[r];
+      sm.lcp[r] = (sa < 0 || sb < 0) ? 0 : min(min(sa, sb) / kPage, kLcpProbe);
+    }
+    __syncthreads();
+    // four compares per thread in flight: all loads first, then the checks
+    const int n_cmp = (B - 1) * kLcpProbe;
+    for (int e0 = tid; e0 < n_cmp; e0 += 4 * NT) {
+      int va[4], vb[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int e = e0 + j * NT, r = 1 + e / kLcpProbe, i = e % kLcpProbe;
+        const bool in = e < n_cmp && i < p.max_pages;
+        va[j] = in ? __ldg(p.block_table + (size_t)(r - 1) * p.max_pages + i) : 0;
+        vb[j] = in ? __ldg(p.block_table + (size_t)r * p.max_pages + i) : 0;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int e = e0 + j * NT, r = 1 + e / kLcpProbe, i = e % kLcpProbe;
+        if (e < n_cmp && va[j] != vb[j] && i < sm.lcp[r]) atomicMin(&sm.lcp[r], i);
+      }
+    }
+    __syncthreads();
     for (int r = warp + 1; r < B; r += kWarps) {
       const int sa = sm.S[r - 1], sb = sm.S[r];
-      if (sa < 0 || sb < 0) continue;
+      if (sa < 0 || sb < 0 || sm.lcp[r] < kLcpProbe) continue;
       const int lim = min(sa, sb) / kPage;  // pages full in both rows
       const int* ba = p.block_table + (size_t)(r - 1) * p.max_pages;
       const int* bb = p.block_table + (size_t)r * p.max_pages;
       // 128 entries per step: four independent loads per lane, then ballots
-      int n = 0;
-      for (int base = 0; base < lim; base += 128) {
+      int n = kLcpProbe;
+      for (int base = kLcpProbe; base < lim; base += 128) {
         bool eq[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -198,12 +233,13 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
         }
         if (stop) break;
       }
+      __syncwarp();
       if (lane == 0) sm.lcp[r] = min(n, lim);
     }
   }
   __syncthreads();
   // group id = (number of run starts up to and including r) - 1
-  for (int r = tid; r < B; r += kPlanThreads)
+  for (int r = tid; r < B; r += NT)
     sm.gid[r] = (r == 0 || !cascade || sm.lcp[r] < kMinSharedPages) ? 1 : 0;
   __syncthreads();
   {
@@ -217,7 +253,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     int total, sum = 0;
 #pragma unroll
     for (int i = 0; i < R; ++i) sum += st[i];
-    int base = cta_scan(sum, &total, sm.sb);
+    int base = cta_scan<NT>(sum, &total, sm.sb);
 #pragma unroll
     for (int i = 0; i < R; ++i) {
       const int r = tid * R + i;
@@ -227,7 +263,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   }
   __syncthreads();
   if (cascade) {
-    for (int r = tid; r < B; r += kPlanThreads) {
+    for (int r = tid; r < B; r += NT) {
       const int g = sm.gid[r];
       if (r > 0 && sm.gid[r - 1] == g) atomicMin(&sm.grp_pages[g], sm.lcp[r]);
       if (sm.kind[r] == 1) {
@@ -238,7 +274,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   }
   __syncthreads();
   // members: decode rows of a group with >= 2 decode rows and a long enough prefix
-  for (int r = tid; r < B; r += kPlanThreads) {
+  for (int r = tid; r < B; r += NT) {
     int m = 0;
     if (cascade && sm.kind[r] == 1) {
       const int g = sm.gid[r];
@@ -248,14 +284,14 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     if (m) sm.flags[r] |= kFlagMember;
   }
   __syncthreads();
-  scan_rows(sm.mrank, B, sm.sb);
-  for (int r = tid; r < B; r += kPlanThreads)
+  scan_rows<NT>(sm.mrank, B, sm.sb);
+  for (int r = tid; r < B; r += NT)
     if (sm.flags[r] & kFlagMember) atomicMin(&sm.grp_base[sm.gid[r]], sm.mrank[r]);
   __syncthreads();
 
   // ---- phase 3: split length
   int w_m = 0, w_lb = 0;
-  for (int r = tid; r < B; r += kPlanThreads) {
+  for (int r = tid; r < B; r += NT) {
     sm.own_pb[r] = 0;
     sm.n_cs[r] = 0;
     sm.sub_first_idx[r] = 0;
@@ -286,8 +322,8 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     w_lb += own + ((sm.flags[r] & kFlagSubFirst) ? gp : 0);
   }
   int tot_wm, tot_wlb;
-  cta_scan(w_m, &tot_wm, sm.sb);
-  cta_scan(w_lb, &tot_wlb, sm.sb);
+  cta_scan<NT>(w_m, &tot_wm, sm.sb);
+  cta_scan<NT>(w_lb, &tot_wlb, sm.sb);
   const int c_bound = max(1, cdiv(tot_wm, kSplitBudget));
   int C;
   if (p.forced_split_pages > 0) {
@@ -299,7 +335,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   }
 
   // ---- phase 4: per-row counts -> offsets
-  for (int r = tid; r < B; r += kPlanThreads) {
+  for (int r = tid; r < B; r += NT) {
     int n_own = 0, n_cs = 0, parts = 0, tiles = 0, sg = 0, direct = 0;
     if (sm.kind[r] == 1) {
       const int pe = cdiv(sm.S[r], kPage);
@@ -320,10 +356,10 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     sm.tile_off[r] = tiles;
   }
   __syncthreads();
-  const int tot_parts = scan_rows(sm.part_off, B, sm.sb);
-  const int tot_items = scan_rows(sm.item_off, B, sm.sb);
-  const int tot_cascade = scan_rows(sm.sg_off, B, sm.sb);
-  const int tot_tiles = scan_rows(sm.tile_off, B, sm.sb);
+  const int tot_parts = scan_rows<NT>(sm.part_off, B, sm.sb);
+  const int tot_items = scan_rows<NT>(sm.item_off, B, sm.sb);
+  const int tot_cascade = scan_rows<NT>(sm.sg_off, B, sm.sb);
+  const int tot_tiles = scan_rows<NT>(sm.tile_off, B, sm.sb);
 
   const bool overflow = tot_items > p.lay.max_decode || tot_cascade > p.lay.max_cascade ||
                         tot_tiles > p.lay.max_append || tot_parts > p.lay.max_parts;
@@ -347,12 +383,12 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   int is_merge_cnt = 0;
   {
     // merge rows get consecutive indices: reuse lcp[] as the scan buffer
-    for (int r = tid; r < B; r += kPlanThreads)
+    for (int r = tid; r < B; r += NT)
       sm.lcp[r] = (sm.kind[r] == 1 && !(sm.flags[r] & kFlagDirect)) ? 1 : 0;
     __syncthreads();
-    is_merge_cnt = scan_rows(sm.lcp, B, sm.sb);
+    is_merge_cnt = scan_rows<NT>(sm.lcp, B, sm.sb);
   }
-  for (int r = tid; r < B; r += kPlanThreads) {
+  for (int r = tid; r < B; r += NT) {
     if (sm.kind[r] != 1) continue;
     const int parts = (r + 1 < B ? sm.part_off[r + 1] : tot_parts) - sm.part_off[r];
     if (!(sm.flags[r] & kFlagDirect)) {
@@ -374,7 +410,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
   }
 
   // ---- phase 6: split records, all threads in parallel
-  for (int e = tid; e < tot_items; e += kPlanThreads) {
+  for (int e = tid; e < tot_items; e += NT) {
     const int r = owner_row(sm.item_off, B, e);
     const int k = e - sm.item_off[r];
     const int S = sm.S[r];
@@ -390,7 +426,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     it.pad = 0;
     ditems[e] = it;
   }
-  for (int e = tid; e < tot_cascade; e += kPlanThreads) {
+  for (int e = tid; e < tot_cascade; e += NT) {
     const int r = owner_row(sm.sg_off, B, e);
     const int k = e - sm.sg_off[r];
     const int gp = sm.grp_pages[sm.gid[r]];
@@ -404,7 +440,7 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
     c.pad0 = c.pad1 = 0;
     citems[e] = c;
   }
-  for (int e = tid; e < tot_tiles; e += kPlanThreads) {
+  for (int e = tid; e < tot_tiles; e += NT) {
     const int r = owner_row(sm.tile_off, B, e);
     const int k = e - sm.tile_off[r];
     const int S = sm.S[r], L = sm.L[r];
@@ -432,18 +468,31 @@ __global__ void __launch_bounds__(kPlanThreads, 1) plan_kernel(AttnParams p) {
 
 cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream) {
   static_assert(sizeof(PlanSmem) < 200 * 1024, "planner shared memory");
-  plan_kernel<<<1, kPlanThreads, sizeof(PlanSmem), stream>>>(p);
+  // fewer threads for small batches: every phase ends in a CTA barrier, and
+  // barriers over 8 warps are cheaper than over 32
+  if (p.num_seqs <= R * 256)
+    plan_kernel<256><<<1, 256, sizeof(PlanSmem), stream>>>(p);
+  else
+    plan_kernel<kPlanThreads><<<1, kPlanThreads, sizeof(PlanSmem), stream>>>(p);
   return cudaGetLastError();
 }
 
 cudaError_t prepare_plan_kernel() {
-  cudaError_t e = cudaFuncSetAttribute(plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(PlanSmem));
-  if (e != cudaSuccess) return e;
   // every kernel of the library asks for the largest shared-memory carveout,
   // so an SM never has to be reconfigured between them and a decode CTA can
   // share an SM with an append CTA
-  return cudaFuncSetAttribute(plan_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                              cudaSharedmemCarveoutMaxShared);
+  cudaError_t e = cudaFuncSetAttribute(plan_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)sizeof(PlanSmem));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(plan_kernel<256>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(plan_kernel<kPlanThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)sizeof(PlanSmem));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(plan_kernel<kPlanThreads>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  return e;
 }
 
 }  // namespace mcpu
