@@ -59,6 +59,8 @@ def _load():
                 P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i64, P, P, i32, P
             ]
             lib.oracle_paged_attention_sampled.restype = ctypes.c_int
+            lib.oracle_rope.argtypes = [P, i64, i32, i32, P, P, i64]
+            lib.oracle_rope.restype = ctypes.c_int
             lib.oracle_double_to_bf16.argtypes = [f64]
             lib.oracle_double_to_bf16.restype = ctypes.c_uint16
             lib.oracle_max_threads.restype = ctypes.c_int
@@ -169,3 +171,28 @@ def bf16_bits_to_float(a) -> np.ndarray:
     """uint16 bf16 bit patterns -> float32 values (exact)."""
     a = np.asarray(a, dtype=np.uint16)
     return (a.astype(np.uint32) << 16).view(np.float32)
+
+
+def token_positions(seq_lens, query_start_loc) -> np.ndarray:
+    """Position of every query token: S_r - L_r + i for token i of row r."""
+    sl = np.asarray(seq_lens, np.int64)
+    qsl = np.asarray(query_start_loc, np.int64)
+    pos = np.zeros(int(qsl[-1]), np.int64)
+    for r in range(len(sl)):
+        L = qsl[r + 1] - qsl[r]
+        pos[qsl[r]:qsl[r + 1]] = sl[r] - L + np.arange(L)
+    return pos
+
+
+def rope(x, positions, cos_sin):
+    """Rotary embedding (step 4) of x [n, heads, D] bf16 bits at the given
+    positions with the table cos_sin [max_position, D]; returns a copy."""
+    lib = _load()
+    x = np.array(x, dtype=np.uint16, copy=True, order="C")
+    pos, pos_p = _c(positions, np.int64)
+    cs, cs_p = _c(cos_sin, np.float32)
+    n, heads, d = x.shape
+    assert cs.shape[1] == d and pos.shape == (n,)
+    rc = lib.oracle_rope(x.ctypes.data_as(ctypes.c_void_p), n, heads, d, pos_p, cs_p, cs.shape[0])
+    _check(rc)
+    return x

@@ -32,6 +32,13 @@
  *         out  = sum_j exp(s_j) / Z * V[j],   lse = ln Z,
  *      evaluated as above with m = max(max_j s_j, sigma_h). sigma_h = -inf
  *      (or no sinks array) is step 2 exactly.
+ *   4. rotary position embedding (optional, before step 1; the rotation of
+ *      q and k that gpt-oss applies, with its angles given as a table): a
+ *      vector x of length D at position p becomes, for i < D/2,
+ *         y_i       = x_i cos_i(p) - x_{i+D/2} sin_i(p)
+ *         y_{i+D/2} = x_{i+D/2} cos_i(p) + x_i sin_i(p)
+ *      with cos_i(p) = table[p][i], sin_i(p) = table[p][D/2 + i] (float),
+ *      products and sums in double, y rounded once to bf16.
  *
  * Precision: bf16 inputs are widened exactly; every sum and product is taken
  * in double; out is rounded once, double -> bf16, to nearest-even.
@@ -325,6 +332,29 @@ int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
     free(acc);
   }
   return err;
+}
+
+/* Step 4 on x [n, heads, D] (bf16 bits, rotated in place): row t sits at
+ * position positions[t]; cos_sin is [max_position, D] float. */
+int oracle_rope(uint16_t* x, int64_t n, int32_t heads, int32_t head_dim, const int64_t* positions,
+                const float* cos_sin, int64_t max_position) {
+  if (n < 0 || heads <= 0 || head_dim <= 0 || head_dim % 2) return ORACLE_ERR_SHAPE;
+  for (int64_t t = 0; t < n; ++t)
+    if (positions[t] < 0 || positions[t] >= max_position) return ORACLE_ERR_LENGTH;
+  const int32_t half = head_dim / 2;
+  for (int64_t t = 0; t < n; ++t) {
+    const float* cs = cos_sin + positions[t] * head_dim;
+    for (int32_t h = 0; h < heads; ++h) {
+      uint16_t* v = x + (t * heads + h) * head_dim;
+      for (int32_t i = 0; i < half; ++i) {
+        double a = bf16_to_double(v[i]), b = bf16_to_double(v[i + half]);
+        double c = (double)cs[i], s = (double)cs[half + i];
+        v[i] = oracle_double_to_bf16(a * c - b * s);
+        v[i + half] = oracle_double_to_bf16(b * c + a * s);
+      }
+    }
+  }
+  return ORACLE_OK;
 }
 
 int oracle_max_threads(void) {

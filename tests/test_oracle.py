@@ -506,3 +506,69 @@ def test_sampled_evaluation_with_sinks_equals_full_evaluation():
                                             h["query_start_loc"], h["sliding_window"], h["softmax_scale"], toks,
                                             heads, sinks=sk)
     assert np.array_equal(so, out[toks, heads]) and np.array_equal(sl, lse[toks, heads])
+
+
+# ------------------------------------------------------ rotary embedding
+
+
+def _rand_bits(shape, seed):
+    x = torch.randn(shape, generator=torch.Generator().manual_seed(seed), dtype=torch.bfloat16)
+    return x.view(torch.int16).numpy().view(np.uint16).copy()
+
+
+def test_rope_with_the_identity_table_changes_nothing():
+    x = _rand_bits((5, 3, 64), 1)
+    tab = np.concatenate([np.ones((10, 32)), np.zeros((10, 32))], axis=1).astype(np.float32)
+    assert np.array_equal(oracle.rope(x, np.array([0, 3, 9, 4, 4]), tab), x)
+
+
+def test_rope_quarter_turn_swaps_halves():
+    x = _rand_bits((4, 2, 64), 2)
+    tab = np.concatenate([np.zeros((8, 32)), np.ones((8, 32))], axis=1).astype(np.float32)
+    y = oracle.rope(x, np.array([1, 2, 3, 7]), tab)
+    assert np.array_equal(y[..., 32:], x[..., :32])
+    neg = (x[..., 32:] ^ 0x8000).astype(np.uint16)  # -x, exact
+    assert np.array_equal(y[..., :32], neg)
+
+
+def test_rope_of_unit_vectors_gives_the_table_entries():
+    tab = W.rope_table(50)
+    x = np.zeros((32, 1, 64), np.uint16)
+    for i in range(32):
+        x[i, 0, i] = 0x3F80  # e_i
+    pos = np.arange(32) + 11
+    y = _f(oracle.rope(x, pos, tab))
+    for i in range(32):
+        c, s = float(tab[pos[i], i]), float(tab[pos[i], 32 + i])
+        assert y[i, 0, i] == _f(np.array([oracle.double_to_bf16(c)]))[0]
+        assert y[i, 0, 32 + i] == _f(np.array([oracle.double_to_bf16(s)]))[0]
+        assert np.count_nonzero(y[i, 0]) <= 2
+
+
+def test_rope_scores_depend_on_relative_position_only():
+    tab = W.rope_table(4096)
+    q = _rand_bits((1, 8, 64), 3)
+    k = _rand_bits((1, 8, 64), 4)
+    base = None
+    for shift in (0, 7, 300, 3000):
+        qr = _f(oracle.rope(q, np.array([40 + shift]), tab))
+        kr = _f(oracle.rope(k, np.array([5 + shift]), tab))
+        s = (qr * kr).sum(axis=-1)[0]
+        bound = 2.0**-7 * (np.linalg.norm(_f(q), axis=-1) * np.linalg.norm(_f(k), axis=-1))[0]
+        if base is None:
+            base = s
+        else:
+            assert np.all(np.abs(s - base) <= bound)
+
+
+def test_rope_preserves_norms():
+    tab = W.rope_table(1000)
+    x = _rand_bits((16, 4, 64), 5)
+    y = oracle.rope(x, np.arange(16) * 61, tab)
+    nx, ny = np.linalg.norm(_f(x), axis=-1), np.linalg.norm(_f(y), axis=-1)
+    assert np.all(np.abs(nx - ny) <= 2.0**-8 * nx)
+
+
+def test_token_positions():
+    pos = oracle.token_positions([10, 4, 7], [0, 1, 1, 4])
+    assert list(pos) == [9, 4, 5, 6]

@@ -442,3 +442,14 @@ def host_rows(batch: Batch, rows, layer: int = 0) -> dict:
         token_map=tok,
         rows=rows,
     )
+
+
+def rope_table(max_position: int, head_dim: int = HEAD_DIM, base: float = 150000.0) -> np.ndarray:
+    """A rotary-embedding table [max_position, head_dim] float32: for position
+    p and i < head_dim / 2, cos(p * base^(-2i/D)) then sin(...). An input of
+    the fused RoPE + KV append (engines precompute it per model); base 150000
+    is gpt-oss's rotary base, without its long-context rescaling."""
+    half = head_dim // 2
+    inv = base ** (-np.arange(half, dtype=np.float64) * 2.0 / head_dim)
+    ang = np.arange(max_position, dtype=np.float64)[:, None] * inv[None, :]
+    return np.concatenate([np.cos(ang), np.sin(ang)], axis=1).astype(np.float32)
