@@ -75,7 +75,8 @@ typedef enum mcpu_status {
   MCPU_ERR_BAD_LENGTHS = 6,          /* device: L_r > S_r, L_r < 0, S_r beyond the table, or
                                         query_start_loc[0] != 0 / [B] != total_q */
   MCPU_ERR_TIMEOUT = 7,              /* device: a bounded wait gave up */
-  MCPU_ERR_INTERNAL = 8              /* device: work plan overflowed its bound */
+  MCPU_ERR_INTERNAL = 8,             /* device: work plan overflowed its bound */
+  MCPU_ERR_POOL_EXHAUSTED = 9        /* device: the free-page stack ran empty */
 } mcpu_status;
 
 typedef struct mcpu_dims {
@@ -193,6 +194,42 @@ mcpu_status mcpu_paged_attention_forward_noalloc(const void* q, const void* k_ca
                                                  const int32_t* query_start_loc, int32_t sliding_window,
                                                  float softmax_scale, const mcpu_dims* dims, void* out,
                                                  float* lse, int32_t* status_word, mcpu_stream_t stream);
+
+/*
+ * KV append with the rotary position embedding fused in (the rotation gpt-oss
+ * applies to q and k before attention; the paper does not describe the
+ * model's layers). For each query token t of row r at position
+ * p = S_r - L_r + i: q[t] (all H_q heads) is rotated in place, and k_new[t]
+ * rotated, v_new[t] as is, are written to (block_table[r][p / 16], p % 16)
+ * exactly as mcpu_kv_append writes them (k_new itself is not modified).
+ * Rotation of a 64-dim row x by table row p, for i < 32:
+ *   y_i = x_i cos_i - x_{i+32} sin_i,  y_{i+32} = x_{i+32} cos_i + x_i sin_i,
+ * cos_i = cos_sin[p * 64 + i], sin_i = cos_sin[p * 64 + 32 + i] (device
+ * float, max_position rows; the caller builds it for its model), computed in
+ * fp32 and rounded once to bf16. Tokens at p >= max_position, or with
+ * inconsistent lengths, set MCPU_ERR_BAD_LENGTHS in status_word and are left
+ * untouched; a bad page skips that token's K/V write (MCPU_ERR_BAD_PAGE).
+ */
+mcpu_status mcpu_rope_kv_append(void* q, const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                                const int32_t* block_table, const int32_t* seq_lens,
+                                const int32_t* query_start_loc, const float* cos_sin, int32_t max_position,
+                                const mcpu_dims* dims, int32_t* status_word, mcpu_stream_t stream);
+
+/*
+ * Grows block tables in place on the device (no host round trip): every
+ * logical page j < ceil(S_r / 16) of row r whose entry block_table[r][j] is
+ * negative receives a page popped from the stack free_pages[0 .. *free_count)
+ * (device int32; the top is free_pages[*free_count - 1]); *free_count is
+ * decremented accordingly. Entries already set (shared prompt pages, pages of
+ * earlier steps) are not touched. Which row gets which popped page is not
+ * specified. If the stack runs empty the remaining entries stay negative and
+ * MCPU_ERR_POOL_EXHAUSTED is raised in status_word. Uses dims->num_seqs and
+ * dims->max_pages_per_seq only. Not a part of the paper's method: the engine
+ * bookkeeping either side of the attention call.
+ */
+mcpu_status mcpu_grow_block_tables(int32_t* block_table, const int32_t* seq_lens, const mcpu_dims* dims,
+                                   const int32_t* free_pages, int32_t* free_count, int32_t* status_word,
+                                   mcpu_stream_t stream);
 
 /* Synchronises `stream`, reads the workspace status word and maps it to the
  * most severe mcpu_status (MCPU_OK if clear). The raw bits go to

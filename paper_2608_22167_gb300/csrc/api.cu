@@ -25,6 +25,14 @@ cudaError_t prepare_append_tc_kernel(int* bpsm);
 cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream);
 cudaError_t prepare_merge_kernel();
 cudaError_t prepare_kv_append_kernel();
+cudaError_t launch_rope_append(void* q, const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                               const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
+                               const float* cos_sin, int32_t max_position, int32_t* status, int32_t num_seqs,
+                               int32_t total_q, int32_t max_pages, int32_t num_pages, int32_t num_q_heads,
+                               int32_t num_kv_heads, cudaStream_t stream);
+cudaError_t launch_grow_tables(int32_t* block_table, const int32_t* seq_lens, int32_t num_seqs, int32_t max_pages,
+                               const int32_t* free_pages, int32_t* free_count, int32_t* status,
+                               cudaStream_t stream);
 cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
                              const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
                              int32_t* status, int32_t num_seqs, int32_t total_q, int32_t max_pages,
@@ -164,6 +172,7 @@ const char* mcpu_status_string(mcpu_status s) {
     case MCPU_ERR_BAD_LENGTHS: return "inconsistent seq_lens / query_start_loc";
     case MCPU_ERR_TIMEOUT: return "device wait timed out";
     case MCPU_ERR_INTERNAL: return "work plan exceeded its bound";
+    case MCPU_ERR_POOL_EXHAUSTED: return "no free KV page left";
   }
   return "unknown status";
 }
@@ -192,6 +201,42 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
   return from_cuda(launch_kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start_loc,
                                     status_word, dims->num_seqs, dims->total_q, dims->max_pages_per_seq,
                                     dims->num_pages, dims->num_kv_heads, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+mcpu_status mcpu_rope_kv_append(void* q, const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                                const int32_t* block_table, const int32_t* seq_lens,
+                                const int32_t* query_start_loc, const float* cos_sin, int32_t max_position,
+                                const mcpu_dims* dims, int32_t* status_word, mcpu_stream_t stream) {
+  mcpu_status st = check_dims(dims);
+  if (st != MCPU_OK) return st;
+  if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
+  if (!q || !k_new || !v_new || !k_cache || !v_cache || !block_table || !seq_lens || !query_start_loc ||
+      !cos_sin || !status_word || max_position < 1)
+    return MCPU_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_cache, 16) ||
+      !aligned(v_cache, 16) || !aligned(cos_sin, 4) || !aligned(status_word, 4))
+    return MCPU_ERR_INVALID_ARG;
+  if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  DeviceState* dev = nullptr;
+  st = device_state(&dev);
+  if (st != MCPU_OK) return st;
+  return from_cuda(launch_rope_append(q, k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start_loc,
+                                      cos_sin, max_position, status_word, dims->num_seqs, dims->total_q,
+                                      dims->max_pages_per_seq, dims->num_pages, dims->num_q_heads,
+                                      dims->num_kv_heads, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+mcpu_status mcpu_grow_block_tables(int32_t* block_table, const int32_t* seq_lens, const mcpu_dims* dims,
+                                   const int32_t* free_pages, int32_t* free_count, int32_t* status_word,
+                                   mcpu_stream_t stream) {
+  if (!dims || dims->num_seqs < 0 || dims->max_pages_per_seq < 0) return MCPU_ERR_INVALID_ARG;
+  if (dims->num_seqs == 0) return MCPU_OK;
+  if (!block_table || !seq_lens || !free_pages || !free_count || !status_word) return MCPU_ERR_INVALID_ARG;
+  if (!aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(free_pages, 4) || !aligned(free_count, 4) ||
+      !aligned(status_word, 4))
+    return MCPU_ERR_INVALID_ARG;
+  return from_cuda(launch_grow_tables(block_table, seq_lens, dims->num_seqs, dims->max_pages_per_seq, free_pages,
+                                      free_count, status_word, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, const void* v_cache,
@@ -320,6 +365,7 @@ mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream,
   if (bits & kStatusBadPage) return MCPU_ERR_BAD_PAGE;
   if (bits & kStatusBadLengths) return MCPU_ERR_BAD_LENGTHS;
   if (bits & kStatusPlanOverflow) return MCPU_ERR_INTERNAL;
+  if (bits & kStatusPoolExhausted) return MCPU_ERR_POOL_EXHAUSTED;
   return MCPU_OK;
 }
 

@@ -33,6 +33,7 @@ constexpr int32_t kStatusBadPage = 1;
 constexpr int32_t kStatusBadLengths = 2;
 constexpr int32_t kStatusTimeout = 4;
 constexpr int32_t kStatusPlanOverflow = 8;
+constexpr int32_t kStatusPoolExhausted = 16;
 
 // Bounded waits: a wait that has not completed after this many nanoseconds
 // of %globaltimer gives up and reports kStatusTimeout.

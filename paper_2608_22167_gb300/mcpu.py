@@ -33,6 +33,7 @@ STATUS = {
     6: "MCPU_ERR_BAD_LENGTHS",
     7: "MCPU_ERR_TIMEOUT",
     8: "MCPU_ERR_INTERNAL",
+    9: "MCPU_ERR_POOL_EXHAUSTED",
 }
 FLAG_NO_CASCADE = 0x1
 FLAG_MMA_SYNC_APPEND = 0x2
@@ -43,6 +44,7 @@ STATUS_BAD_PAGE = 1
 STATUS_BAD_LENGTHS = 2
 STATUS_TIMEOUT = 4
 STATUS_PLAN_OVERFLOW = 8
+STATUS_POOL_EXHAUSTED = 16
 
 
 class McpuError(RuntimeError):
@@ -90,6 +92,10 @@ _lib.mcpu_paged_attention_forward_noalloc.argtypes = [
     _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P, _P,
 ]
 _lib.mcpu_paged_attention_forward_noalloc.restype = ctypes.c_int
+_lib.mcpu_rope_kv_append.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.POINTER(Dims), _P, _P]
+_lib.mcpu_rope_kv_append.restype = ctypes.c_int
+_lib.mcpu_grow_block_tables.argtypes = [_P, _P, ctypes.POINTER(Dims), _P, _P, _P, _P]
+_lib.mcpu_grow_block_tables.restype = ctypes.c_int
 _lib.mcpu_read_device_status.argtypes = [_P, _P, ctypes.POINTER(ctypes.c_int32)]
 _lib.mcpu_read_device_status.restype = ctypes.c_int
 _lib.mcpu_reset_device_status.argtypes = [_P, _P]
@@ -166,6 +172,34 @@ def mcpu_kv_append(k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_
                             _ptr(seq_lens), _ptr(query_start_loc), ctypes.byref(d), _ptr(status_word),
                             _stream(stream)),
         "mcpu_kv_append",
+    )
+
+
+def mcpu_rope_kv_append(q, k_new, v_new, k_cache, v_cache, block_table, seq_lens, query_start_loc, cos_sin,
+                        status_word, stream=None):
+    """Rotates q in place and writes rotated k_new / v_new into the pools;
+    cos_sin: float32 device tensor [max_position, 64] (cos then sin)."""
+    if cos_sin.dtype != torch.float32 or cos_sin.dim() != 2 or cos_sin.shape[1] != q.shape[2]:
+        raise ValueError("cos_sin must be a float32 [max_position, head_dim] tensor")
+    d = dims(q, k_cache, block_table, seq_lens)
+    _check(
+        _lib.mcpu_rope_kv_append(_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(block_table),
+                                 _ptr(seq_lens), _ptr(query_start_loc), _ptr(cos_sin), int(cos_sin.shape[0]),
+                                 ctypes.byref(d), _ptr(status_word), _stream(stream)),
+        "mcpu_rope_kv_append",
+    )
+
+
+def mcpu_grow_block_tables(block_table, seq_lens, free_pages, free_count, status_word, stream=None):
+    """Fills every negative block-table entry a row needs for its seq_len with
+    a page popped from the device stack free_pages[0:free_count] (int32
+    tensors; free_count is a one-element device tensor, decremented)."""
+    d = Dims(num_seqs=int(seq_lens.shape[0]), total_q=0, max_pages_per_seq=int(block_table.shape[1]), num_pages=0,
+             num_q_heads=1, num_kv_heads=1, head_dim=64, page_size=16)
+    _check(
+        _lib.mcpu_grow_block_tables(_ptr(block_table), _ptr(seq_lens), ctypes.byref(d), _ptr(free_pages),
+                                    _ptr(free_count), _ptr(status_word), _stream(stream)),
+        "mcpu_grow_block_tables",
     )
 
 

@@ -120,7 +120,7 @@ def test_kv_append_host_validation(lib):
 def test_status_strings(lib):
     lib.mcpu_status_string.restype = ctypes.c_char_p
     seen = set()
-    for code in range(9):
+    for code in range(10):
         s = lib.mcpu_status_string(code)
         assert s and s not in seen
         seen.add(s)
