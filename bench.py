@@ -771,8 +771,8 @@ def main():
                     help="host-only simulator steps before the churn workload's first GPU step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--launch", choices=["graph", "eager"], default="eager",
-                    help="time eager C-ABI calls (default) or CUDA-graph replays of the whole step")
+    ap.add_argument("--launch", choices=["graph", "eager"], default="graph",
+                    help="time CUDA-graph replays of the whole step (default) or eager C-ABI calls")
     ap.add_argument("--no-compare-launch", dest="compare_launch", action="store_false",
                     help="skip timing the other launch mode")
     args = ap.parse_args()
