@@ -59,6 +59,20 @@ def _load():
                 P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i64, P, P, i32, P
             ]
             lib.oracle_paged_attention_sampled.restype = ctypes.c_int
+            lib.oracle_paged_attention_fp8.argtypes = [
+                P, P, P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i32, P
+            ]
+            lib.oracle_paged_attention_fp8.restype = ctypes.c_int
+            lib.oracle_paged_attention_sampled_fp8.argtypes = [
+                P, P, P, P, P, P, P, P, i32, i32, i64, i32, i32, i32, i32, i32, f64, P, P, i64, P, P, i32, P
+            ]
+            lib.oracle_paged_attention_sampled_fp8.restype = ctypes.c_int
+            lib.oracle_kv_append_fp8.argtypes = [P, P, P, P, P, P, P, P, P, i32, i32, i64, i32, i32, i32]
+            lib.oracle_kv_append_fp8.restype = ctypes.c_int
+            lib.oracle_e4m3_to_double.argtypes = [ctypes.c_uint8]
+            lib.oracle_e4m3_to_double.restype = f64
+            lib.oracle_float_to_e4m3.argtypes = [ctypes.c_float]
+            lib.oracle_float_to_e4m3.restype = ctypes.c_uint8
             lib.oracle_rope.argtypes = [P, i64, i32, i32, P, P, i64]
             lib.oracle_rope.restype = ctypes.c_int
             lib.oracle_double_to_bf16.argtypes = [f64]
@@ -196,3 +210,90 @@ def rope(x, positions, cos_sin):
     rc = lib.oracle_rope(x.ctypes.data_as(ctypes.c_void_p), n, heads, d, pos_p, cs_p, cs.shape[0])
     _check(rc)
     return x
+
+
+# ------------------------------------------------------------ fp8 pages (step 5)
+
+
+def e4m3_to_float(code: int) -> float:
+    return float(_load().oracle_e4m3_to_double(int(code)))
+
+
+def float_to_e4m3(x: float) -> int:
+    return int(_load().oracle_float_to_e4m3(float(x)))
+
+
+def kv_append_fp8(k_new, v_new, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc, page_size=16):
+    """Copies of the fp8 pools (codes uint8 [P, Hkv, page, D]) and scales
+    (float32 [P, Hkv, page]) with the new rows quantized and written in."""
+    lib = _load()
+    k8 = np.array(k8, dtype=np.uint8, copy=True, order="C")
+    v8 = np.array(v8, dtype=np.uint8, copy=True, order="C")
+    ks = np.array(k_scale, dtype=np.float32, copy=True, order="C")
+    vs = np.array(v_scale, dtype=np.float32, copy=True, order="C")
+    kn, kn_p = _c(k_new, np.uint16)
+    vn, vn_p = _c(v_new, np.uint16)
+    bt, bt_p = _c(block_table, np.int32)
+    sl, sl_p = _c(seq_lens, np.int32)
+    qs, qs_p = _c(query_start_loc, np.int32)
+    num_pages, hkv, page, d = k8.shape
+    assert page == page_size
+    P = ctypes.c_void_p
+    rc = lib.oracle_kv_append_fp8(kn_p, vn_p, k8.ctypes.data_as(P), v8.ctypes.data_as(P), ks.ctypes.data_as(P),
+                                  vs.ctypes.data_as(P), bt_p, sl_p, qs_p, sl.shape[0], bt.shape[1], num_pages, hkv,
+                                  d, page)
+    _check(rc)
+    return k8, v8, ks, vs
+
+
+def paged_attention_fp8(q, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc, sliding_window,
+                        softmax_scale, num_threads=0, sinks=None):
+    """Attention over fp8 pools: (out bf16 bits, lse)."""
+    lib = _load()
+    q, q_p = _c(q, np.uint16)
+    k8, k8_p = _c(k8, np.uint8)
+    v8, v8_p = _c(v8, np.uint8)
+    ks, ks_p = _c(k_scale, np.float32)
+    vs, vs_p = _c(v_scale, np.float32)
+    bt, bt_p = _c(block_table, np.int32)
+    sl, sl_p = _c(seq_lens, np.int32)
+    qs, qs_p = _c(query_start_loc, np.int32)
+    T, hq, d = q.shape
+    num_pages, hkv, page, _ = k8.shape
+    sk, sk_p = _sinks(sinks, hq)
+    out = np.zeros((T, hq, d), np.uint16)
+    lse = np.zeros((T, hq), np.float32)
+    rc = lib.oracle_paged_attention_fp8(q_p, k8_p, v8_p, ks_p, vs_p, bt_p, sl_p, qs_p, sl.shape[0], bt.shape[1],
+                                        num_pages, hq, hkv, d, page, int(sliding_window), float(softmax_scale),
+                                        out.ctypes.data_as(ctypes.c_void_p), lse.ctypes.data_as(ctypes.c_void_p),
+                                        int(num_threads), sk_p)
+    _check(rc)
+    return out, lse
+
+
+def paged_attention_sampled_fp8(q, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc,
+                                sliding_window, softmax_scale, tokens, heads, num_threads=0, sinks=None):
+    lib = _load()
+    q, q_p = _c(q, np.uint16)
+    k8, k8_p = _c(k8, np.uint8)
+    v8, v8_p = _c(v8, np.uint8)
+    ks, ks_p = _c(k_scale, np.float32)
+    vs, vs_p = _c(v_scale, np.float32)
+    bt, bt_p = _c(block_table, np.int32)
+    sl, sl_p = _c(seq_lens, np.int32)
+    qs, qs_p = _c(query_start_loc, np.int32)
+    tk, tk_p = _c(tokens, np.int64)
+    hd, hd_p = _c(heads, np.int32)
+    T, hq, d = q.shape
+    num_pages, hkv, page, _ = k8.shape
+    n = tk.shape[0]
+    sk, sk_p = _sinks(sinks, hq)
+    out = np.zeros((n, d), np.uint16)
+    lse = np.zeros((n,), np.float32)
+    rc = lib.oracle_paged_attention_sampled_fp8(q_p, k8_p, v8_p, ks_p, vs_p, bt_p, sl_p, qs_p, sl.shape[0],
+                                                bt.shape[1], num_pages, hq, hkv, d, page, int(sliding_window),
+                                                float(softmax_scale), tk_p, hd_p, n,
+                                                out.ctypes.data_as(ctypes.c_void_p),
+                                                lse.ctypes.data_as(ctypes.c_void_p), int(num_threads), sk_p)
+    _check(rc)
+    return out, lse

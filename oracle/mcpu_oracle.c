@@ -39,6 +39,15 @@
  *         y_{i+D/2} = x_{i+D/2} cos_i(p) + x_i sin_i(p)
  *      with cos_i(p) = table[p][i], sin_i(p) = table[p][D/2 + i] (float),
  *      products and sums in double, y rounded once to bf16.
+ *   5. fp8 KV pages (optional; a storage variant, not in the paper): each new
+ *      (token, kv head) row x of 64 bf16 values is stored as 64 e4m3 codes
+ *      and one float scale. In float arithmetic: a = max_i |x_i|; if a = 0
+ *      the codes and the scale are 0, else inv = 448 / a, scale = a / 448
+ *      and code_i = e4m3(x_i * inv), the nearest e4m3 value (ties to even,
+ *      saturating at +-448). e4m3 here is the "fn" format: 1 sign, 4
+ *      exponent (bias 7), 3 mantissa bits, subnormals down to 2^-9, largest
+ *      448, no infinities. Attention then reads K[j][d] = e4m3value(code) *
+ *      scale (in double) in place of the bf16 value.
  *
  * Precision: bf16 inputs are widened exactly; every sum and product is taken
  * in double; out is rounded once, double -> bf16, to nearest-even.
@@ -158,6 +167,92 @@ int oracle_kv_append(const uint16_t* k_new, const uint16_t* v_new, uint16_t* k_c
   return ORACLE_OK;
 }
 
+/* Step 5: value of an e4m3 code. */
+double oracle_e4m3_to_double(uint8_t c) {
+  int e = (c >> 3) & 15, m = c & 7;
+  if (e == 15 && m == 7) return NAN;
+  double v = e == 0 ? ldexp((double)m, -9) : ldexp((double)(8 + m), e - 10);
+  return (c & 0x80) ? -v : v;
+}
+
+/* Step 5: nearest e4m3 code of a float, ties to even, saturating at 448.
+ * The quantum of the binade [2^e, 2^(e+1)) is 2^(e-3) (subnormals: 2^-9). */
+uint8_t oracle_float_to_e4m3(float x) {
+  if (isnan(x)) return 0x7F;
+  uint8_t sign = signbit(x) ? 0x80 : 0;
+  double a = fabs((double)x);
+  if (a >= 448.0) return sign | 0x7E;
+  if (a == 0.0) return sign;
+  int ex;
+  frexp(a, &ex); /* a = f 2^ex, 0.5 <= f < 1 */
+  int e = ex - 1;
+  if (e < -6) e = -6;
+  double q = ldexp(1.0, e - 3);
+  double r = rint(a / q) * q; /* a / q is exact: q is a power of two */
+  if (r == 0.0) return sign;
+  if (r >= 448.0) return sign | 0x7E;
+  if (r < ldexp(1.0, -6)) return sign | (uint8_t)(r / ldexp(1.0, -9)); /* subnormal */
+  frexp(r, &ex);
+  int E = ex - 1;
+  int m = (int)(r / ldexp(1.0, E - 3)) - 8;
+  return sign | (uint8_t)(((E + 7) << 3) | m);
+}
+
+/* Step 5 for one row of n bf16 values: codes and the scale. */
+static void quantize_row(const uint16_t* x, int32_t n, uint8_t* codes, float* scale) {
+  float a = 0.f;
+  for (int32_t i = 0; i < n; ++i) {
+    float v = (float)fabs(bf16_to_double(x[i]));
+    if (v > a) a = v;
+  }
+  if (a == 0.f) {
+    for (int32_t i = 0; i < n; ++i) codes[i] = 0;
+    *scale = 0.f;
+    return;
+  }
+  volatile float inv = 448.0f / a; /* float arithmetic, as defined */
+  *scale = a / 448.0f;
+  for (int32_t i = 0; i < n; ++i) {
+    volatile float y = (float)bf16_to_double(x[i]) * inv;
+    codes[i] = oracle_float_to_e4m3(y);
+  }
+}
+
+/* Step 1 with step 5: scatter the quantized new rows into fp8 pools
+ * k8/v8 [num_pages, H_kv, page, D] and scales [num_pages, H_kv, page]. */
+int oracle_kv_append_fp8(const uint16_t* k_new, const uint16_t* v_new, uint8_t* k8, uint8_t* v8,
+                         float* k_scale, float* v_scale, const int32_t* block_table,
+                         const int32_t* seq_lens, const int32_t* query_start_loc, int32_t num_seqs,
+                         int32_t max_pages_per_seq, int64_t num_pages, int32_t num_kv_heads,
+                         int32_t head_dim, int32_t page_size) {
+  int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_kv_heads,
+                        num_kv_heads, head_dim, page_size);
+  if (rc) return rc;
+  for (int32_t r = 0; r < num_seqs; ++r) {
+    int64_t L = query_start_loc[r + 1] - query_start_loc[r];
+    int64_t S = seq_lens[r];
+    for (int64_t i = 0; i < L; ++i) {
+      int64_t page = block_table[(int64_t)r * max_pages_per_seq + (S - L + i) / page_size];
+      if (page < 0 || page >= num_pages) return ORACLE_ERR_PAGE;
+    }
+  }
+  for (int32_t r = 0; r < num_seqs; ++r) {
+    int64_t L = query_start_loc[r + 1] - query_start_loc[r];
+    int64_t S = seq_lens[r];
+    for (int64_t i = 0; i < L; ++i) {
+      int64_t tok = query_start_loc[r] + i;
+      int64_t pos = S - L + i;
+      int64_t page = block_table[(int64_t)r * max_pages_per_seq + pos / page_size];
+      for (int32_t h = 0; h < num_kv_heads; ++h) {
+        int64_t row = (page * num_kv_heads + h) * page_size + pos % page_size;
+        quantize_row(k_new + (tok * num_kv_heads + h) * head_dim, head_dim, k8 + row * head_dim, k_scale + row);
+        quantize_row(v_new + (tok * num_kv_heads + h) * head_dim, head_dim, v8 + row * head_dim, v_scale + row);
+      }
+    }
+  }
+  return ORACLE_OK;
+}
+
 /* Visible key range [lo, p] of a query at position p (step 2's mask). */
 static int64_t first_visible(int64_t p, int32_t window) {
   if (window <= 0) return 0;
@@ -165,9 +260,23 @@ static int64_t first_visible(int64_t p, int32_t window) {
   return lo < 0 ? 0 : lo;
 }
 
+/* Where K and V come from: bf16 pools (step 2), or fp8 pools with their
+ * per-row scales (step 5). Rows are (page * H_kv + kv head) * page + slot. */
+typedef struct {
+  const uint16_t *k16, *v16;
+  const uint8_t *k8, *v8;
+  const float *ks, *vs;
+} kv_src;
+
+static double kv_value(const kv_src* src, int is_v, int64_t row, int32_t d, int32_t head_dim) {
+  if (src->k16) return bf16_to_double((is_v ? src->v16 : src->k16)[row * head_dim + d]);
+  return oracle_e4m3_to_double((is_v ? src->v8 : src->k8)[row * head_dim + d]) *
+         (double)(is_v ? src->vs : src->ks)[row];
+}
+
 /* Step 2 for one query vector: gathers its visible keys straight from the
  * pages and writes out[0..D) (bf16 bits) and *lse. */
-static int attend_one(const uint16_t* qv, const uint16_t* k_cache, const uint16_t* v_cache,
+static int attend_one(const uint16_t* qv, const kv_src* src,
                       const int32_t* bt_row, int64_t p, int32_t kvh, int32_t window,
                       double scale, double sink, int64_t num_pages, int32_t num_kv_heads,
                       int32_t head_dim, int32_t page_size, double* s, double* acc, uint16_t* out,
@@ -184,9 +293,9 @@ static int attend_one(const uint16_t* qv, const uint16_t* k_cache, const uint16_
   for (int64_t j = lo; j <= p; ++j) {
     int64_t page = bt_row[j / page_size];
     if (page < 0 || page >= num_pages) return ORACLE_ERR_PAGE;
-    const uint16_t* kj = k_cache + ((page * num_kv_heads + kvh) * page_size + j % page_size) * head_dim;
+    const int64_t kr = (page * num_kv_heads + kvh) * page_size + j % page_size;
     double dot = 0.0;
-    for (int32_t d = 0; d < head_dim; ++d) dot += bf16_to_double(qv[d]) * bf16_to_double(kj[d]);
+    for (int32_t d = 0; d < head_dim; ++d) dot += bf16_to_double(qv[d]) * kv_value(src, 0, kr, d, head_dim);
     s[j - lo] = scale * dot;
     if (s[j - lo] > m) m = s[j - lo];
   }
@@ -199,9 +308,9 @@ static int attend_one(const uint16_t* qv, const uint16_t* k_cache, const uint16_
   for (int32_t d = 0; d < head_dim; ++d) acc[d] = 0.0;
   for (int64_t j = lo; j <= p; ++j) {
     int64_t page = bt_row[j / page_size];
-    const uint16_t* vj = v_cache + ((page * num_kv_heads + kvh) * page_size + j % page_size) * head_dim;
+    const int64_t vr = (page * num_kv_heads + kvh) * page_size + j % page_size;
     double w = exp(s[j - lo] - m) / l;
-    for (int32_t d = 0; d < head_dim; ++d) acc[d] += w * bf16_to_double(vj[d]);
+    for (int32_t d = 0; d < head_dim; ++d) acc[d] += w * kv_value(src, 1, vr, d, head_dim);
   }
   for (int32_t d = 0; d < head_dim; ++d) out[d] = oracle_double_to_bf16(acc[d]);
   *lse = (float)(m + log(l));
@@ -214,15 +323,14 @@ static int row_of_token(const int32_t* qsl, int32_t num_seqs, int64_t t) {
   return -1;
 }
 
-/* Full attention: every query token of every row, every q head.
- * num_threads <= 0 uses the OpenMP default. */
-int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
-                           const int32_t* block_table, const int32_t* seq_lens,
-                           const int32_t* query_start_loc, int32_t num_seqs,
-                           int32_t max_pages_per_seq, int64_t num_pages, int32_t num_q_heads,
-                           int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
-                           int32_t sliding_window, double softmax_scale, uint16_t* out,
-                           float* lse, int32_t num_threads, const float* sinks) {
+/* Full attention: every query token of every row, every q head. */
+static int paged_attention_impl(const uint16_t* q, const kv_src* src,
+                                const int32_t* block_table, const int32_t* seq_lens,
+                                const int32_t* query_start_loc, int32_t num_seqs,
+                                int32_t max_pages_per_seq, int64_t num_pages, int32_t num_q_heads,
+                                int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
+                                int32_t sliding_window, double softmax_scale, uint16_t* out,
+                                float* lse, int32_t num_threads, const float* sinks) {
   int rc = check_common(seq_lens, query_start_loc, num_seqs, max_pages_per_seq, num_q_heads,
                         num_kv_heads, head_dim, page_size);
   if (rc) return rc;
@@ -253,7 +361,7 @@ int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uin
         int64_t S = seq_lens[r];
         int64_t L = query_start_loc[r + 1] - query_start_loc[r];
         int64_t p = S - L + (t - query_start_loc[r]);
-        int e = attend_one(q + (t * num_q_heads + h) * head_dim, k_cache, v_cache,
+        int e = attend_one(q + (t * num_q_heads + h) * head_dim, src,
                            block_table + (int64_t)r * max_pages_per_seq, p, h / group,
                            sliding_window, softmax_scale, sinks ? (double)sinks[h] : -INFINITY,
                            num_pages, num_kv_heads, head_dim, page_size, s, acc,
@@ -270,11 +378,9 @@ int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uin
   return err;
 }
 
-/* The same definition evaluated only at listed (token, q head) pairs, for
- * spot checks of workloads too large to run in full. out_samples is
- * [n_samples, D] bf16 bits, lse_samples [n_samples]. */
-int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
-                                   const uint16_t* v_cache, const int32_t* block_table,
+/* The same at listed (token, q head) pairs. */
+static int paged_attention_sampled_impl(const uint16_t* q, const kv_src* src,
+                                   const int32_t* block_table,
                                    const int32_t* seq_lens, const int32_t* query_start_loc,
                                    int32_t num_seqs, int32_t max_pages_per_seq, int64_t num_pages,
                                    int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
@@ -318,7 +424,7 @@ int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
       int64_t S = seq_lens[r];
       int64_t L = query_start_loc[r + 1] - query_start_loc[r];
       int64_t p = S - L + (t - query_start_loc[r]);
-      int e = attend_one(q + (t * num_q_heads + h) * head_dim, k_cache, v_cache,
+      int e = attend_one(q + (t * num_q_heads + h) * head_dim, src,
                          block_table + (int64_t)r * max_pages_per_seq, p, h / group,
                          sliding_window, softmax_scale, sinks ? (double)sinks[h] : -INFINITY,
                          num_pages, num_kv_heads, head_dim, page_size, s, acc,
@@ -355,6 +461,69 @@ int oracle_rope(uint16_t* x, int64_t n, int32_t heads, int32_t head_dim, const i
     }
   }
   return ORACLE_OK;
+}
+
+/* Full attention (steps 2-3) over bf16 pools. num_threads <= 0 uses the
+ * OpenMP default. */
+int oracle_paged_attention(const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
+                           const int32_t* block_table, const int32_t* seq_lens,
+                           const int32_t* query_start_loc, int32_t num_seqs,
+                           int32_t max_pages_per_seq, int64_t num_pages, int32_t num_q_heads,
+                           int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
+                           int32_t sliding_window, double softmax_scale, uint16_t* out,
+                           float* lse, int32_t num_threads, const float* sinks) {
+  kv_src src = {k_cache, v_cache, NULL, NULL, NULL, NULL};
+  return paged_attention_impl(q, &src, block_table, seq_lens, query_start_loc, num_seqs, max_pages_per_seq,
+                              num_pages, num_q_heads, num_kv_heads, head_dim, page_size, sliding_window,
+                              softmax_scale, out, lse, num_threads, sinks);
+}
+
+/* The same over fp8 pools with per-row scales (step 5). */
+int oracle_paged_attention_fp8(const uint16_t* q, const uint8_t* k8, const uint8_t* v8, const float* k_scale,
+                               const float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
+                               const int32_t* query_start_loc, int32_t num_seqs, int32_t max_pages_per_seq,
+                               int64_t num_pages, int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                               int32_t page_size, int32_t sliding_window, double softmax_scale, uint16_t* out,
+                               float* lse, int32_t num_threads, const float* sinks) {
+  kv_src src = {NULL, NULL, k8, v8, k_scale, v_scale};
+  return paged_attention_impl(q, &src, block_table, seq_lens, query_start_loc, num_seqs, max_pages_per_seq,
+                              num_pages, num_q_heads, num_kv_heads, head_dim, page_size, sliding_window,
+                              softmax_scale, out, lse, num_threads, sinks);
+}
+
+/* The definition evaluated only at listed (token, q head) pairs, for spot
+ * checks of workloads too large to run in full. out_samples is
+ * [n_samples, D] bf16 bits, lse_samples [n_samples]. */
+int oracle_paged_attention_sampled(const uint16_t* q, const uint16_t* k_cache,
+                                   const uint16_t* v_cache, const int32_t* block_table,
+                                   const int32_t* seq_lens, const int32_t* query_start_loc,
+                                   int32_t num_seqs, int32_t max_pages_per_seq, int64_t num_pages,
+                                   int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                   int32_t page_size, int32_t sliding_window,
+                                   double softmax_scale, const int64_t* sample_token,
+                                   const int32_t* sample_head, int64_t n_samples,
+                                   uint16_t* out_samples, float* lse_samples,
+                                   int32_t num_threads, const float* sinks) {
+  kv_src src = {k_cache, v_cache, NULL, NULL, NULL, NULL};
+  return paged_attention_sampled_impl(q, &src, block_table, seq_lens, query_start_loc, num_seqs,
+                                      max_pages_per_seq, num_pages, num_q_heads, num_kv_heads, head_dim,
+                                      page_size, sliding_window, softmax_scale, sample_token, sample_head,
+                                      n_samples, out_samples, lse_samples, num_threads, sinks);
+}
+
+int oracle_paged_attention_sampled_fp8(const uint16_t* q, const uint8_t* k8, const uint8_t* v8,
+                                       const float* k_scale, const float* v_scale, const int32_t* block_table,
+                                       const int32_t* seq_lens, const int32_t* query_start_loc, int32_t num_seqs,
+                                       int32_t max_pages_per_seq, int64_t num_pages, int32_t num_q_heads,
+                                       int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
+                                       int32_t sliding_window, double softmax_scale, const int64_t* sample_token,
+                                       const int32_t* sample_head, int64_t n_samples, uint16_t* out_samples,
+                                       float* lse_samples, int32_t num_threads, const float* sinks) {
+  kv_src src = {NULL, NULL, k8, v8, k_scale, v_scale};
+  return paged_attention_sampled_impl(q, &src, block_table, seq_lens, query_start_loc, num_seqs,
+                                      max_pages_per_seq, num_pages, num_q_heads, num_kv_heads, head_dim,
+                                      page_size, sliding_window, softmax_scale, sample_token, sample_head,
+                                      n_samples, out_samples, lse_samples, num_threads, sinks);
 }
 
 int oracle_max_threads(void) {

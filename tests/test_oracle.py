@@ -572,3 +572,140 @@ def test_rope_preserves_norms():
 def test_token_positions():
     pos = oracle.token_positions([10, 4, 7], [0, 1, 1, 4])
     assert list(pos) == [9, 4, 5, 6]
+
+
+# ------------------------------------------------------------ fp8 KV pages
+
+
+def _torch_e4m3(xs):
+    """torch's float32 -> float8_e4m3fn conversion (round to nearest even)."""
+    t = torch.from_numpy(np.asarray(xs, np.float32)).to(torch.float8_e4m3fn)
+    return t.view(torch.uint8).numpy()
+
+
+def test_e4m3_decoding_matches_torch_for_all_codes():
+    codes = np.arange(256, dtype=np.uint8)
+    ref = torch.from_numpy(codes).view(torch.float8_e4m3fn).float().numpy().astype(np.float64)
+    got = np.array([oracle.e4m3_to_float(c) for c in codes])
+    nan = np.isnan(ref)
+    assert np.array_equal(nan, np.isnan(got)) and np.array_equal(np.nonzero(nan)[0], [0x7F, 0xFF])
+    assert np.array_equal(got[~nan], ref[~nan])
+    # format facts: largest 448, smallest subnormal 2^-9, smallest normal 2^-6
+    assert got[0x7E] == 448.0 and got[0x01] == 2.0**-9 and got[0x08] == 2.0**-6 and got[0xFE] == -448.0
+
+
+def test_e4m3_encoding_round_trips_every_code():
+    for c in range(256):
+        if c & 0x7F == 0x7F:
+            continue
+        assert oracle.float_to_e4m3(oracle.e4m3_to_float(c)) == c
+
+
+def test_e4m3_encoding_matches_torch_in_range():
+    rng = np.random.default_rng(21)
+    mags = np.concatenate([
+        rng.uniform(0, 464, 3000),
+        np.exp2(rng.uniform(-14, 9, 3000)),
+        rng.uniform(0, 2.0**-6, 1000),  # subnormal range
+    ])
+    mags = mags[mags <= 464]
+    xs = (mags * rng.choice([-1.0, 1.0], mags.size)).astype(np.float32)
+    got = np.array([oracle.float_to_e4m3(float(x)) for x in xs], np.uint8)
+    assert np.array_equal(got, _torch_e4m3(xs))
+
+
+def test_e4m3_encoding_ties_go_to_the_even_code():
+    vals = np.array([oracle.e4m3_to_float(c) for c in range(0x7F)])
+    mids = ((vals[:-1] + vals[1:]) / 2).astype(np.float32)  # exact in float32
+    got = np.array([oracle.float_to_e4m3(float(m)) for m in mids], np.uint8)
+    lo = np.arange(0x7E, dtype=np.uint8)
+    assert np.array_equal(got, np.where(lo % 2 == 0, lo, lo + 1))
+    assert np.array_equal(got, _torch_e4m3(mids))
+
+
+def test_e4m3_encoding_saturates():
+    for x in [448.0, 449.0, 464.0, 465.0, 1e6, 3.0e38, math.inf]:
+        assert oracle.float_to_e4m3(x) == 0x7E and oracle.float_to_e4m3(-x) == 0xFE
+    assert oracle.float_to_e4m3(math.nan) & 0x7F == 0x7F
+    assert oracle.float_to_e4m3(2.0**-11) == 0 and oracle.float_to_e4m3(-0.0) == 0x80
+
+
+def _fp8_pools(num_pages, hkv, page, d):
+    return (np.zeros((num_pages, hkv, page, d), np.uint8), np.zeros((num_pages, hkv, page, d), np.uint8),
+            np.zeros((num_pages, hkv, page), np.float32), np.zeros((num_pages, hkv, page), np.float32))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_kv_append_fp8_quantizes_each_row_by_its_absmax(seed):
+    b = W.fuzz_batch(500 + seed)
+    h = W.host_inputs(b)
+    num_pages, hkv, page, d = h["k_cache"].shape
+    k8, v8, ks, vs = oracle.kv_append_fp8(h["k_new"], h["v_new"], *_fp8_pools(num_pages, hkv, page, d),
+                                          h["block_table"], h["seq_lens"], h["query_start_loc"])
+    qsl, sl, bt = h["query_start_loc"], h["seq_lens"], h["block_table"]
+    written = np.zeros((num_pages, hkv, page), bool)
+    for r in range(len(sl)):
+        L, S = int(qsl[r + 1] - qsl[r]), int(sl[r])
+        for i in range(L):
+            t, pos = int(qsl[r]) + i, S - L + i
+            pg, slot = int(bt[r, pos // page]), pos % page
+            for kvh in range(hkv):
+                written[pg, kvh, slot] = True
+                for src, codes, scale in ((h["k_new"], k8, ks), (h["v_new"], v8, vs)):
+                    x = oracle.bf16_bits_to_float(src[t, kvh]).astype(np.float32)
+                    a = np.float32(np.abs(x).max())
+                    if a == 0:
+                        assert scale[pg, kvh, slot] == 0 and not codes[pg, kvh, slot].any()
+                        continue
+                    assert scale[pg, kvh, slot] == a / np.float32(448)
+                    want = _torch_e4m3(x * (np.float32(448) / a))
+                    assert np.array_equal(codes[pg, kvh, slot], want)
+                    assert (want[np.argmax(np.abs(x))] & 0x7F) == 0x7E  # the absmax maps to +-448
+                    deq = np.array([oracle.e4m3_to_float(c) for c in want]) * float(scale[pg, kvh, slot])
+                    err = np.abs(deq - x.astype(np.float64))
+                    # half a quantum: 2^-4 relative for normals, 2^-10 * scale below 2^-6 * scale
+                    assert np.all(err <= np.abs(x) * 2.0**-4 * (1 + 1e-6) + float(scale[pg, kvh, slot]) * 2.0**-10)
+    assert not k8[~written].any() and not v8[~written].any()
+    assert not ks[~written].any() and not vs[~written].any()
+
+
+def _exact_fp8_batch(seed):
+    """A batch whose bf16 pools hold e4m3 values times a power-of-two scale
+    per row, so that the fp8 pools describe the very same K and V."""
+    b = W.fuzz_batch(seed)
+    h = W.host_inputs(b)
+    num_pages, hkv, page, d = h["k_cache"].shape
+    rng = np.random.default_rng(seed)
+    pools = []
+    for _ in range(2):
+        codes = rng.integers(0, 256, size=(num_pages, hkv, page, d)).astype(np.uint8)
+        codes[(codes & 0x7F) == 0x7F] = 0x3A
+        scale = np.exp2(rng.integers(-8, -2, size=(num_pages, hkv, page))).astype(np.float32)
+        vals = np.array([oracle.e4m3_to_float(c) for c in range(256)])[codes] * scale[..., None]
+        bits = torch.from_numpy(vals.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy()
+        assert np.array_equal(oracle.bf16_bits_to_float(bits.view(np.uint16)), vals)  # exact in bf16
+        pools.append((codes, scale, bits.view(np.uint16)))
+    return h, pools
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_fp8_attention_equals_bf16_attention_on_the_same_values(seed):
+    h, ((k8, ks, k16), (v8, vs, v16)) = _exact_fp8_batch(600 + seed)
+    args = (h["block_table"], h["seq_lens"], h["query_start_loc"], h["sliding_window"], h["softmax_scale"])
+    sk = _sinks(h["q"].shape[1], seed) if seed % 2 else None
+    o8, l8 = oracle.paged_attention_fp8(h["q"], k8, v8, ks, vs, *args, sinks=sk)
+    o16, l16 = oracle.paged_attention(h["q"], k16, v16, *args, sinks=sk)
+    assert np.array_equal(o8, o16) and np.array_equal(l8, l16)
+    ref_out, ref_lse = brute.attention(h["q"], k16, v16, *args, sinks=sk)
+    _assert_close_to_exact(o8, l8, ref_out, ref_lse)
+
+
+def test_sampled_fp8_evaluation_equals_full_evaluation():
+    h, ((k8, ks, _), (v8, vs, _)) = _exact_fp8_batch(610)
+    args = (h["block_table"], h["seq_lens"], h["query_start_loc"], h["sliding_window"], h["softmax_scale"])
+    out, lse = oracle.paged_attention_fp8(h["q"], k8, v8, ks, vs, *args)
+    rng = np.random.default_rng(4)
+    toks = rng.integers(0, out.shape[0], size=24).astype(np.int64)
+    heads = rng.integers(0, h["q"].shape[1], size=24).astype(np.int32)
+    so, sl = oracle.paged_attention_sampled_fp8(h["q"], k8, v8, ks, vs, *args, toks, heads)
+    assert np.array_equal(so, out[toks, heads]) and np.array_equal(sl, lse[toks, heads])
