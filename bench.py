@@ -89,6 +89,11 @@ DECODE_SOURCES = [
     "paper_2608_22167_gb300/csrc/decode.cu",
     "paper_2608_22167_gb300/csrc/common.cuh",
 ]
+FP8_SOURCES = [
+    "paper_2608_22167_gb300/csrc/fp8.cu",
+    "paper_2608_22167_gb300/csrc/common.cuh",
+]
+FP8_WORKLOADS = ("tiny", "decode", "long")
 
 
 def peaks():
@@ -123,7 +128,15 @@ def whole_job_gbs(bytes_per_rank: int, world: int, ms: float) -> float:
 # --------------------------------------------------------------- accounting
 
 
-def layer_stats(batch: W.Batch, layer: int):
+def kv_token_bytes(batch: W.Batch, kv: str = "bf16") -> int:
+    """KV bytes one token occupies over all kv heads: bf16 K and V rows, or
+    e4m3 codes plus one float scale per row."""
+    if kv == "fp8":
+        return 2 * batch.num_kv_heads * (batch.head_dim + 4)
+    return KV_TOKEN_BYTES(batch)
+
+
+def layer_stats(batch: W.Batch, layer: int, kv: str = "bf16"):
     """Algorithmic work of one layer: KV bytes (distinct visible tokens, shared
     prompt pages once per group), attended (query, key) pairs, split by
     decode / append rows."""
@@ -155,7 +168,7 @@ def layer_stats(batch: W.Batch, layer: int):
             while n < lim and all(bt[r, n] == ref[n] for r in rows):
                 n += 1
             shared_tokens += (len(rows) - 1) * n * batch.page_size
-    tb = KV_TOKEN_BYTES(batch)
+    tb = kv_token_bytes(batch, kv)
     dec = L == 1
     app = L > 1
     return dict(
@@ -283,6 +296,58 @@ class Stepper:
         return sum(self.launches_per_layer.values())
 
 
+def quantize_pools_fp8(batch: W.Batch, dev):
+    """fp8 copies of every pool, written by mcpu_kv_append_fp8 with every
+    page appended as one 16-token row (input preparation, untimed)."""
+    from paper_2608_22167_gb300 import mcpu
+
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    pools = {}
+    for key, pool in batch.pools.items():
+        P, H, page, D = pool.k_cache.shape
+        k8 = torch.empty((P, H, page, D), dtype=torch.uint8, device=dev)
+        v8 = torch.empty((P, H, D, page), dtype=torch.uint8, device=dev)
+        ks = torch.empty((P, H, page), dtype=torch.float32, device=dev)
+        vs = torch.empty_like(ks)
+        chunk = 2048  # rows per call (the planner's row limit)
+        for p0 in range(0, P, chunk):
+            n = min(chunk, P - p0)
+            kn = pool.k_cache[p0:p0 + n].permute(0, 2, 1, 3).reshape(n * page, H, D).contiguous()
+            vn = pool.v_cache[p0:p0 + n].permute(0, 2, 1, 3).reshape(n * page, H, D).contiguous()
+            bt = torch.arange(p0, p0 + n, dtype=torch.int32, device=dev).view(n, 1)
+            sl = torch.full((n,), page, dtype=torch.int32, device=dev)
+            qsl = torch.arange(0, (n + 1) * page, page, dtype=torch.int32, device=dev)
+            mcpu.mcpu_kv_append_fp8(kn, vn, k8, v8, ks, vs, bt, sl, qsl, status)
+        pools[key] = (k8, v8, ks, vs)
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"fp8 pool quantization: device status {int(status.item())}")
+    return pools
+
+
+class Fp8Stepper(Stepper):
+    """The same step over fp8 KV pages: quantizing KV append, then the fp8
+    forward (decode rows only)."""
+
+    def __init__(self, batch: W.Batch, dev):
+        super().__init__(batch, dev)
+        self.pools8 = quantize_pools_fp8(batch, dev)
+        for i, lay in enumerate(batch.layers):
+            self.launches_per_layer[i] = 4 + (1 if lay.sliding_window <= 0 else 0)  # append, plan, decode, [cascade], merge
+
+    def layer_call(self, i, q=None, k_new=None, v_new=None, out=None, lse=None, events=None):
+        m = self.mcpu
+        lay = self.layers[i]
+        k8, v8, ks, vs = self.pools8[lay.pool]
+        bt = self.bts[lay.pool]
+        m.mcpu_kv_append_fp8(lay.k_new if k_new is None else k_new, lay.v_new if v_new is None else v_new,
+                             k8, v8, ks, vs, bt, self.sl, self.qsl, m.status_word(self.ws))
+        m.mcpu_paged_attention_forward_fp8(lay.q if q is None else q, k8, v8, ks, vs, bt, self.sl, self.qsl,
+                                           lay.sliding_window, self.batch.softmax_scale,
+                                           self.out if out is None else out, self.lse if lse is None else lse,
+                                           self.ws, phase_events=events)
+
+
 def make_batch(name, dev, rank):
     fn = W.CONFIGS[name]
     seed = {"tiny": 1001, "decode": 1002, "mixed": 1003, "mixed_small": 1013, "long": 1004,
@@ -290,7 +355,20 @@ def make_batch(name, dev, rank):
     return fn(seed=seed, device=dev)
 
 
-def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int):
+def oracle_fp8_pools(k_bits, v_bits):
+    """A (compact, host) bf16 pool quantized by the oracle, every page
+    appended as one 16-token row: (k8, v8, k_scale, v_scale), V row-major."""
+    import oracle
+
+    P, H, page, D = k_bits.shape
+    tok = lambda x: np.ascontiguousarray(x.transpose(0, 2, 1, 3).reshape(P * page, H, D))  # noqa: E731
+    z8 = np.zeros((P, H, page, D), np.uint8)
+    zs = np.zeros((P, H, page), np.float32)
+    return oracle.kv_append_fp8(tok(k_bits), tok(v_bits), z8, z8, zs, zs, np.arange(P, dtype=np.int32)[:, None],
+                                np.full(P, page, np.int32), np.arange(P + 1, dtype=np.int32) * page)
+
+
+def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int, kv: str = "bf16"):
     """Time the oracle on a bounded sample of the workload and scale its
     throughput to the whole step by attended (query, key) pairs."""
     import oracle
@@ -310,8 +388,12 @@ def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int):
         if len(app):
             rows += list(rng.choice(app, size=min(2, len(app)), replace=False))
         h = W.host_rows(batch, rows, 0)
-        kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
-                                  h["seq_lens"], h["query_start_loc"])
+        if kv == "fp8":
+            pools8 = oracle.kv_append_fp8(h["k_new"], h["v_new"], *oracle_fp8_pools(h["k_cache"], h["v_cache"]),
+                                          h["block_table"], h["seq_lens"], h["query_start_loc"])
+        else:
+            kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                                      h["seq_lens"], h["query_start_loc"])
         qsl = h["query_start_loc"]
         toks = []
         for i in range(len(h["rows"])):
@@ -330,8 +412,12 @@ def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int):
         p = S - Lr + (toks - qsl[row_of])
         vis = p + 1 if Wn <= 0 else np.minimum(p + 1, Wn)
         t = time.perf_counter()
-        oracle.paged_attention_sampled(h["q"], kc, vc, h["block_table"], h["seq_lens"], qsl, Wn,
-                                       batch.softmax_scale, tk, hd)
+        if kv == "fp8":
+            oracle.paged_attention_sampled_fp8(h["q"], *pools8, h["block_table"], h["seq_lens"], qsl, Wn,
+                                               batch.softmax_scale, tk, hd)
+        else:
+            oracle.paged_attention_sampled(h["q"], kc, vc, h["block_table"], h["seq_lens"], qsl, Wn,
+                                           batch.softmax_scale, tk, hd)
         t_spent += time.perf_counter() - t
         pairs_done += int(vis.sum()) * batch.num_q_heads
         n_tok += len(toks)
@@ -342,7 +428,8 @@ def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int):
         unit="GB/s",
         cores=int(oracle.max_threads()),
         kind="oracle",
-        sample=f"{n_tok} query tokens x {batch.num_q_heads} heads from {rounds} draws of 6 decode + 2 append "
+        sample=f"{'fp8 pages, ' if kv == 'fp8' else ''}"
+               f"{n_tok} query tokens x {batch.num_q_heads} heads from {rounds} draws of 6 decode + 2 append "
                f"rows (layer 0), {t_spent:.1f} s of oracle time; step time scaled by attended (query, key) pairs "
                f"({pairs_done:.3g} of {pairs_total:.3g})",
         est_step_ms=est_step_s * 1e3,
@@ -354,9 +441,12 @@ def run_ours(args, rank, world, dev):
     from paper_2608_22167_gb300 import mcpu
 
     hbm, tc_burst, tc_sust, peak_src = peaks()
+    fp8 = args.kv == "fp8"
+    if fp8 and args.workload not in FP8_WORKLOADS:
+        raise SystemExit(f"--kv fp8 runs decode-only workloads: {', '.join(FP8_WORKLOADS)}")
     batch = make_batch(args.workload, dev, rank)
-    st = Stepper(batch, dev)
-    per_layer = [layer_stats(batch, i) for i in range(len(batch.layers))]
+    st = Fp8Stepper(batch, dev) if fp8 else Stepper(batch, dev)
+    per_layer = [layer_stats(batch, i, args.kv) for i in range(len(batch.layers))]
     kv_bytes = sum(s["kv_bytes"] for s in per_layer)
     pairs = sum(s["pairs"] for s in per_layer)
 
@@ -460,8 +550,11 @@ def run_ours(args, rank, world, dev):
             ktime["plan"] += t[1]
             ktime["decode"] += t[2] - t[1]
             ktime["cascade"] += t[3] - t[2]
-            ktime["append_chunk"] += t[4] - t[1]
-            ktime["merge"] += t[5] - max(t[3], t[4])
+            if fp8:  # one stream, no append kernel: [3] and [4] coincide
+                ktime["merge"] += t[5] - t[4]
+            else:
+                ktime["append_chunk"] += t[4] - t[1]
+                ktime["merge"] += t[5] - max(t[3], t[4])
     ktime = {n: v / n_sets for n, v in ktime.items()}
     dec_bytes = sum(s["kv_bytes"] - s["kv_bytes_append"] for s in per_layer)
     app_flops = sum(s["flops_append"] for s in per_layer)
@@ -472,12 +565,16 @@ def run_ours(args, rank, world, dev):
         ach = dec_bytes / (dec_ms * 1e-3) / 1e9
         traffic = None
         if args.workload in ("decode", "long"):
-            traffic = recorded_traffic("decode_kernel_decode_long.md", f"traffic_bytes_per_launch_{args.workload}",
-                                       DECODE_SOURCES)
+            if fp8:
+                traffic = recorded_traffic("decode_fp8_kernel_decode_long.md",
+                                           f"traffic_bytes_per_launch_{args.workload}", FP8_SOURCES)
+            else:
+                traffic = recorded_traffic("decode_kernel_decode_long.md",
+                                           f"traffic_bytes_per_launch_{args.workload}", DECODE_SOURCES)
         roof_dec = {"bound": "hbm", "achieved": round(ach, 1), "peak": hbm, "unit": "GB/s",
                     "frac": round(ach / hbm, 4), "traffic": traffic,
-                    "kernel": "decode_kernel (+cascade pass)", "peak_source": f"{peak_src} hbm_gbs",
-                    "ms_per_step": round(dec_ms, 4)}
+                    "kernel": ("decode_fp8_kernel" if fp8 else "decode_kernel") + " (+cascade pass)",
+                    "peak_source": f"{peak_src} hbm_gbs", "ms_per_step": round(dec_ms, 4)}
     roof_app = None
     if app_ms > 0 and app_flops > 0:
         ach = app_flops / (app_ms * 1e-3) / 1e12
@@ -557,10 +654,12 @@ def run_ours(args, rank, world, dev):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) bf16 Q/K/V; lengths drawn per the workload recipe)",
+        "dtype": "e4m3 KV pages (f16 MMA, f32 softmax), bf16 q/out" if fp8 else "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V; lengths drawn per the workload recipe)"
+                + ("; the pools quantized to e4m3 with one scale per (token, kv head) row" if fp8 else ""),
         "config": {
-            "workload": WORKLOAD_DESC[args.workload],
+            "workload": ("fp8 KV pages, " if fp8 else "") + WORKLOAD_DESC[args.workload],
+            "kv": args.kv,
             "layers": nl,
             "rows": batch.num_seqs,
             "query_tokens": batch.total_q,
@@ -588,7 +687,7 @@ def run_ours(args, rank, world, dev):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         stats0 = per_layer[0]
         cb = cpu_baseline_sample(batch, {"kv_bytes": stats0["kv_bytes"], "pairs": stats0["pairs"]},
-                                 args.cpu_seconds, seed=99)
+                                 args.cpu_seconds, seed=99, kv=args.kv)
         res["cpu_baseline"] = {k: (round(v, 4) if isinstance(v, float) else v) for k, v in cb.items()}
     return res
 
@@ -726,16 +825,18 @@ def run_reference(args, rank, world):
     """The oracle (plain CPU definition) timed on the host cores, rank 0 only."""
     if rank != 0:
         return None
+    if args.kv == "fp8" and args.workload not in FP8_WORKLOADS:
+        raise SystemExit(f"--kv fp8 runs decode-only workloads: {', '.join(FP8_WORKLOADS)}")
     batch = make_batch(args.workload, "cuda" if torch.cuda.is_available() else "cpu", 0)
-    stats0 = layer_stats(batch, 0)
+    stats0 = layer_stats(batch, 0, args.kv)
     nl = len(batch.layers)
     per_step = max(2.0, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
     for w in range(args.warmup):
-        cpu_baseline_sample(batch, stats0, per_step / 4, seed=1000 + w)
+        cpu_baseline_sample(batch, stats0, per_step / 4, seed=1000 + w, kv=args.kv)
     vals, ms = [], []
     cb = None
     for k in range(args.steps):
-        cb = cpu_baseline_sample(batch, stats0, per_step, seed=2000 + k)
+        cb = cpu_baseline_sample(batch, stats0, per_step, seed=2000 + k, kv=args.kv)
         vals.append(cb["value"])
         ms.append(cb["est_step_ms"] * nl)
     value = float(statistics.mean(vals))
@@ -752,7 +853,8 @@ def run_reference(args, rank, world):
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic (seeded N(0,1) bf16 Q/K/V; lengths drawn per the workload recipe)",
-        "config": {"workload": WORKLOAD_DESC[args.workload], "layers": nl, "rows": batch.num_seqs},
+        "config": {"workload": ("fp8 KV pages, " if args.kv == "fp8" else "") + WORKLOAD_DESC[args.workload],
+                   "kv": args.kv, "layers": nl, "rows": batch.num_seqs},
         "impl": "reference",
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cb["cores"], "kind": "oracle",
                          "sample": cb["sample"]},
@@ -769,6 +871,8 @@ def main():
     ap.add_argument("--workload", choices=sorted(W.CONFIGS) + ["churn"], default="mixed")
     ap.add_argument("--churn-settle", type=int, default=400,
                     help="host-only simulator steps before the churn workload's first GPU step")
+    ap.add_argument("--kv", choices=["bf16", "fp8"], default="bf16",
+                    help="KV page format; fp8 (e4m3 + per-row scales) runs decode-only workloads")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--launch", choices=["graph", "eager"], default="graph",

@@ -76,7 +76,9 @@ typedef enum mcpu_status {
                                         query_start_loc[0] != 0 / [B] != total_q */
   MCPU_ERR_TIMEOUT = 7,              /* device: a bounded wait gave up */
   MCPU_ERR_INTERNAL = 8,             /* device: work plan overflowed its bound */
-  MCPU_ERR_POOL_EXHAUSTED = 9        /* device: the free-page stack ran empty */
+  MCPU_ERR_POOL_EXHAUSTED = 9,       /* device: the free-page stack ran empty */
+  MCPU_ERR_UNSUPPORTED_ROW = 10      /* device: a row the called variant does not handle was
+                                        skipped (an append row given to the fp8 forward) */
 } mcpu_status;
 
 typedef struct mcpu_dims {
@@ -230,6 +232,51 @@ mcpu_status mcpu_rope_kv_append(void* q, const void* k_new, const void* v_new, v
 mcpu_status mcpu_grow_block_tables(int32_t* block_table, const int32_t* seq_lens, const mcpu_dims* dims,
                                    const int32_t* free_pages, int32_t* free_count, int32_t* status_word,
                                    mcpu_stream_t stream);
+
+/*
+ * fp8 KV pages (a storage variant for the memory-bound decode; not in the
+ * paper, which keeps K/V in bf16). Each (token, kv head) row x of D = 64
+ * values is stored as 64 e4m3 codes (OCP "e4m3fn": bias 7, largest 448,
+ * subnormals down to 2^-9, no infinities) and one float scale, computed in
+ * float arithmetic as a = max_i |x_i|, scale = a / 448,
+ * code_i = e4m3(x_i * (448 / a)) rounded to nearest-even and saturated to
+ * +-448 (an all-zero row stores zero codes and scale 0). Attention reads
+ * K[j][d] = value(code) * scale. One scale per row rather than per page, so
+ * that a page can fill one token at a time without requantizing.
+ *
+ * Layouts (device memory, 16-byte aligned):
+ *   k8       [num_pages, H_kv, 16, D] uint8  codes, one 64-byte row per key
+ *   v8       [num_pages, H_kv, D, 16] uint8  codes, each (page, kv head)
+ *            block TRANSPOSED: v8[page][h][d][slot]
+ *   k_scale, v_scale [num_pages, H_kv, 16] float
+ * Slots of a page that no row has written may hold anything: the kernels
+ * mask them (their codes become finite numbers that are multiplied by 0).
+ *
+ * mcpu_kv_append_fp8: as mcpu_kv_append (same placement, lengths and error
+ * bits), quantizing each new row as above; k_new, v_new stay bf16.
+ */
+mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
+                               float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
+                               const int32_t* query_start_loc, const mcpu_dims* dims, int32_t* status_word,
+                               mcpu_stream_t stream);
+
+/*
+ * mcpu_paged_attention_forward over fp8 pages, for decode rows (L_r = 1 or
+ * 0): same arguments, results and options as mcpu_paged_attention_forward
+ * (split-KV, cascade pass over shared prompt pages, sliding window, sinks,
+ * phase events, graph capture), with the pools replaced by the four fp8
+ * arrays. dims->num_pages counts pages of k8 (and v8). A batch with
+ * total_q > num_seqs (some row appends) returns MCPU_ERR_UNSUPPORTED
+ * without launching; an append row found on the device is skipped and
+ * reported as MCPU_ERR_UNSUPPORTED_ROW. MCPU_FLAG_MMA_SYNC_APPEND is not
+ * accepted; every kernel runs on `stream`.
+ */
+mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* k8, const void* v8, const float* k_scale,
+                                             const float* v_scale, const int32_t* block_table,
+                                             const int32_t* seq_lens, const int32_t* query_start_loc,
+                                             int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
+                                             void* out, float* lse, void* workspace, size_t workspace_bytes,
+                                             const mcpu_options* opts, mcpu_stream_t stream);
 
 /* Synchronises `stream`, reads the workspace status word and maps it to the
  * most severe mcpu_status (MCPU_OK if clear). The raw bits go to

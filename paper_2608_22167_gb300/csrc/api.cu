@@ -37,6 +37,13 @@ cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache
                              const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
                              int32_t* status, int32_t num_seqs, int32_t total_q, int32_t max_pages,
                              int32_t num_pages, int32_t num_kv_heads, cudaStream_t stream);
+cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
+                                 float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
+                                 const int32_t* qsl, int32_t* status, int32_t num_seqs, int32_t total_q,
+                                 int32_t max_pages, int32_t num_pages, int32_t num_kv_heads, cudaStream_t stream);
+cudaError_t launch_decode_fp8(const void* k8, const void* v8, const float* k_scale, const float* v_scale,
+                              const AttnParams& p, int grid, bool cascade, cudaStream_t stream);
+cudaError_t prepare_fp8_kernels(int* bpsm_decode, int* bpsm_cascade);
 }  // namespace mcpu
 
 namespace {
@@ -49,6 +56,7 @@ struct DeviceState {
   bool ready = false;
   int sms = 0;
   int bpsm_decode = 0, bpsm_cascade = 0, bpsm_append = 0, bpsm_append_tc = 0;
+  int bpsm_fp8 = 0, bpsm_fp8_cascade = 0;
   // side stream for the memory-bound decode kernels, and the fork/join events
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
@@ -92,7 +100,9 @@ mcpu_status device_state(DeviceState** out) {
     if ((e = prepare_append_tc_kernel(&st.bpsm_append_tc)) != cudaSuccess) return cuda_fail(e);
     if ((e = prepare_merge_kernel()) != cudaSuccess) return cuda_fail(e);
     if ((e = prepare_kv_append_kernel()) != cudaSuccess) return cuda_fail(e);
-    if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1 || st.bpsm_append_tc < 1)
+    if ((e = prepare_fp8_kernels(&st.bpsm_fp8, &st.bpsm_fp8_cascade)) != cudaSuccess) return cuda_fail(e);
+    if (st.bpsm_decode < 1 || st.bpsm_cascade < 1 || st.bpsm_append < 1 || st.bpsm_append_tc < 1 ||
+        st.bpsm_fp8 < 1 || st.bpsm_fp8_cascade < 1)
       return MCPU_ERR_CUDA;
     int lo_prio = 0, hi_prio = 0;
     if ((e = cudaDeviceGetStreamPriorityRange(&lo_prio, &hi_prio)) != cudaSuccess) return cuda_fail(e);
@@ -157,7 +167,7 @@ mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : cuda_
 
 extern "C" {
 
-int32_t mcpu_abi_version(void) { return 2; }
+int32_t mcpu_abi_version(void) { return 3; }
 
 int32_t mcpu_last_cuda_error(void) { return t_last_cuda_error; }
 
@@ -173,6 +183,7 @@ const char* mcpu_status_string(mcpu_status s) {
     case MCPU_ERR_TIMEOUT: return "device wait timed out";
     case MCPU_ERR_INTERNAL: return "work plan exceeded its bound";
     case MCPU_ERR_POOL_EXHAUSTED: return "no free KV page left";
+    case MCPU_ERR_UNSUPPORTED_ROW: return "a row this variant does not handle was skipped";
   }
   return "unknown status";
 }
@@ -295,6 +306,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   p.oob_row = (int32_t)rows;
   p.append_tile_tok = (legacy_append ? kAppendRowsMin : kAppendTcRows) / p.group;
   p.sinks = opts ? opts->sinks : nullptr;
+  p.decode_only = 0;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   void* const* ev = opts ? opts->phase_events : nullptr;
@@ -354,6 +366,117 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   return from_cuda(e);
 }
 
+mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
+                               float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
+                               const int32_t* query_start_loc, const mcpu_dims* dims, int32_t* status_word,
+                               mcpu_stream_t stream) {
+  mcpu_status st = check_dims(dims);
+  if (st != MCPU_OK) return st;
+  if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
+  if (!k_new || !v_new || !k8 || !v8 || !k_scale || !v_scale || !block_table || !seq_lens || !query_start_loc ||
+      !status_word)
+    return MCPU_ERR_INVALID_ARG;
+  if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k8, 16) || !aligned(v8, 16) || !aligned(k_scale, 16) ||
+      !aligned(v_scale, 16) || !aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(query_start_loc, 4) ||
+      !aligned(status_word, 4))
+    return MCPU_ERR_INVALID_ARG;
+  if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  DeviceState* dev = nullptr;
+  st = device_state(&dev);
+  if (st != MCPU_OK) return st;
+  return from_cuda(launch_kv_append_fp8(k_new, v_new, k8, v8, k_scale, v_scale, block_table, seq_lens,
+                                        query_start_loc, status_word, dims->num_seqs, dims->total_q,
+                                        dims->max_pages_per_seq, dims->num_pages, dims->num_kv_heads,
+                                        reinterpret_cast<cudaStream_t>(stream)));
+}
+
+mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* k8, const void* v8, const float* k_scale,
+                                             const float* v_scale, const int32_t* block_table,
+                                             const int32_t* seq_lens, const int32_t* query_start_loc,
+                                             int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
+                                             void* out, float* lse, void* workspace, size_t workspace_bytes,
+                                             const mcpu_options* opts, mcpu_stream_t stream) {
+  mcpu_status st = check_dims(dims);
+  if (st != MCPU_OK) return st;
+  if (!(softmax_scale > 0.f) || softmax_scale > 3.0e38f) return MCPU_ERR_INVALID_ARG;
+  if (!workspace) return MCPU_ERR_INVALID_ARG;
+  if (workspace_bytes < mcpu_workspace_size(dims)) return MCPU_ERR_WORKSPACE_TOO_SMALL;
+  if (!aligned(workspace, 256)) return MCPU_ERR_INVALID_ARG;
+  if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
+  // decode rows only: more query tokens than rows means some row appends
+  if (dims->total_q > dims->num_seqs) return MCPU_ERR_UNSUPPORTED;
+  if (!q || !k8 || !v8 || !k_scale || !v_scale || !block_table || !seq_lens || !query_start_loc || !out || !lse)
+    return MCPU_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(k8, 16) || !aligned(v8, 16) || !aligned(k_scale, 16) || !aligned(v_scale, 16) ||
+      !aligned(out, 16) || !aligned(lse, 4) || !aligned(block_table, 4) || !aligned(seq_lens, 4) ||
+      !aligned(query_start_loc, 4))
+    return MCPU_ERR_INVALID_ARG;
+  if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  if (opts && opts->split_pages < 0) return MCPU_ERR_INVALID_ARG;
+  if (opts && opts->sinks && !aligned(opts->sinks, 4)) return MCPU_ERR_INVALID_ARG;
+  if (opts && (opts->flags & MCPU_FLAG_MMA_SYNC_APPEND)) return MCPU_ERR_UNSUPPORTED;
+
+  DeviceState* dev = nullptr;
+  st = device_state(&dev);
+  if (st != MCPU_OK) return st;
+
+  AttnParams p;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.block_table = block_table;
+  p.seq_lens = seq_lens;
+  p.qsl = query_start_loc;
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.lse = lse;
+  p.ws = static_cast<uint8_t*>(workspace);
+  p.num_seqs = dims->num_seqs;
+  p.total_q = dims->total_q;
+  p.max_pages = dims->max_pages_per_seq;
+  p.num_pages = dims->num_pages;
+  p.num_q_heads = dims->num_q_heads;
+  p.num_kv_heads = dims->num_kv_heads;
+  p.group = dims->num_q_heads / dims->num_kv_heads;
+  p.lay = workspace_layout(p.num_seqs, p.total_q, p.num_q_heads, p.group);
+  p.window = sliding_window > 0 ? sliding_window : 0;
+  p.scale_log2 = softmax_scale * 1.4426950408889634f;
+  p.total_warps_hint = dev->sms * dev->bpsm_fp8 * 4;
+  p.forced_split_pages = opts ? opts->split_pages : 0;
+  p.cascade_enabled = (opts && (opts->flags & MCPU_FLAG_NO_CASCADE)) ? 0 : 1;
+  p.oob_row = 0;
+  p.append_tile_tok = kAppendTcRows / p.group;
+  p.sinks = opts ? opts->sinks : nullptr;
+  p.decode_only = 1;
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  void* const* ev = opts ? opts->phase_events : nullptr;
+  cudaStreamCaptureStatus capturing = cudaStreamCaptureStatusNone;
+  if (ev) {
+    const cudaError_t ce = cudaStreamIsCapturing(s, &capturing);
+    if (ce != cudaSuccess) return cuda_fail(ce);
+  }
+  const unsigned int rec_flags = capturing == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : 0u;
+  auto mark = [&](int i) -> cudaError_t {
+    return ev ? cudaEventRecordWithFlags(reinterpret_cast<cudaEvent_t>(ev[i]), s, rec_flags) : cudaSuccess;
+  };
+  const bool cascade = p.cascade_enabled && p.window == 0;
+  // every kernel on `stream`: there is no append kernel to run beside
+  cudaError_t e = mark(0);
+  if (e == cudaSuccess) e = launch_plan(p, s);
+  if (e == cudaSuccess) e = mark(1);
+  if (e == cudaSuccess) e = launch_decode_fp8(k8, v8, k_scale, v_scale, p, dev->sms * dev->bpsm_fp8, false, s);
+  if (e == cudaSuccess) e = mark(2);
+  if (e == cudaSuccess && cascade)
+    e = launch_decode_fp8(k8, v8, k_scale, v_scale, p, dev->sms * dev->bpsm_fp8_cascade, true, s);
+  if (e == cudaSuccess) e = mark(3);
+  if (e == cudaSuccess) e = mark(4);
+  if (e == cudaSuccess) {
+    const int want = (p.num_seqs * p.num_q_heads + 7) / 8;
+    const int grid = want < dev->sms * 8 ? (want > 0 ? want : 1) : dev->sms * 8;
+    e = launch_merge(p, grid, s);
+  }
+  if (e == cudaSuccess) e = mark(5);
+  return from_cuda(e);
+}
+
 mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream, int32_t* status_bits) {
   if (!workspace) return MCPU_ERR_INVALID_ARG;
   int32_t bits = 0;
@@ -366,6 +489,7 @@ mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream,
   if (bits & kStatusBadLengths) return MCPU_ERR_BAD_LENGTHS;
   if (bits & kStatusPlanOverflow) return MCPU_ERR_INTERNAL;
   if (bits & kStatusPoolExhausted) return MCPU_ERR_POOL_EXHAUSTED;
+  if (bits & kStatusUnsupportedRow) return MCPU_ERR_UNSUPPORTED_ROW;
   return MCPU_OK;
 }
 

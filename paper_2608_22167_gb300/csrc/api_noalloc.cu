@@ -173,6 +173,7 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
   p.oob_row = (int32_t)rows;
   p.append_tile_tok = kAppendTcRows / group;
   p.sinks = nullptr;
+  p.decode_only = 0;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // The scratch keeps the previous call's contents: the status word must

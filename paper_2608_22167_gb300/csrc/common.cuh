@@ -34,6 +34,7 @@ constexpr int32_t kStatusBadLengths = 2;
 constexpr int32_t kStatusTimeout = 4;
 constexpr int32_t kStatusPlanOverflow = 8;
 constexpr int32_t kStatusPoolExhausted = 16;
+constexpr int32_t kStatusUnsupportedRow = 32;  // a row the called variant does not handle (skipped)
 
 // Bounded waits: a wait that has not completed after this many nanoseconds
 // of %globaltimer gives up and reports kStatusTimeout.
@@ -124,6 +125,7 @@ struct AttnParams {
   int32_t oob_row;               // y coordinate just past the pool, read as zeros
   int32_t append_tile_tok;       // tokens per append tile (tile rows / group)
   const float* sinks;            // [Hq] sink logits (natural log), or null
+  int32_t decode_only;           // 1: rows with L > 1 are reported and skipped (fp8 pools)
 };
 
 // Attention sinks (gpt-oss): q head h has a logit sigma_h that joins the
@@ -250,6 +252,27 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
       "{%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// The same with fp16 inputs.
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                              uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Untiled bulk copy global -> shared (16-byte aligned addresses, size a
+// multiple of 16), completion signalled on the mbarrier as transaction bytes.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
+                                          uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::
+          "r"(dst),
+      "l"(src), "r"(bytes), "r"(bar), "l"(policy)
+      : "memory");
 }
 
 // Transpose of an 8x8 matrix of 16-bit elements held one row-pair per lane.

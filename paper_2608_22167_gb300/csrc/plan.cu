@@ -159,10 +159,13 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
     const int len = q1 - q0, s = p.seq_lens[r];
     const bool bad = len < 0 || s < len || s > p.max_pages * kPage;
     if (bad) atomicOr(&hdr->status, kStatusBadLengths);
-    sm.S[r] = bad ? -1 : s;
-    sm.L[r] = bad ? 0 : len;
+    // decode-only calls (fp8 pools) report and skip append rows
+    const bool skip = !bad && p.decode_only && len > 1;
+    if (skip) atomicOr(&hdr->status, kStatusUnsupportedRow);
+    sm.S[r] = (bad || skip) ? -1 : s;
+    sm.L[r] = (bad || skip) ? 0 : len;
     sm.Q0[r] = q0;
-    sm.kind[r] = bad ? 0 : (len == 0 ? 0 : (len == 1 ? 1 : 2));
+    sm.kind[r] = (bad || skip) ? 0 : (len == 0 ? 0 : (len == 1 ? 1 : 2));
     sm.lcp[r] = 0;
     sm.grp_pages[r] = 0x7fffffff;
     sm.grp_ndec[r] = 0;

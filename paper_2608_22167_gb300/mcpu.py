@@ -34,6 +34,7 @@ STATUS = {
     7: "MCPU_ERR_TIMEOUT",
     8: "MCPU_ERR_INTERNAL",
     9: "MCPU_ERR_POOL_EXHAUSTED",
+    10: "MCPU_ERR_UNSUPPORTED_ROW",
 }
 FLAG_NO_CASCADE = 0x1
 FLAG_MMA_SYNC_APPEND = 0x2
@@ -45,6 +46,7 @@ STATUS_BAD_LENGTHS = 2
 STATUS_TIMEOUT = 4
 STATUS_PLAN_OVERFLOW = 8
 STATUS_POOL_EXHAUSTED = 16
+STATUS_UNSUPPORTED_ROW = 32
 
 
 class McpuError(RuntimeError):
@@ -96,6 +98,13 @@ _lib.mcpu_rope_kv_append.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.
 _lib.mcpu_rope_kv_append.restype = ctypes.c_int
 _lib.mcpu_grow_block_tables.argtypes = [_P, _P, ctypes.POINTER(Dims), _P, _P, _P, _P]
 _lib.mcpu_grow_block_tables.restype = ctypes.c_int
+_lib.mcpu_kv_append_fp8.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.POINTER(Dims), _P, _P]
+_lib.mcpu_kv_append_fp8.restype = ctypes.c_int
+_lib.mcpu_paged_attention_forward_fp8.argtypes = [
+    _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P,
+    ctypes.c_size_t, ctypes.POINTER(Options), _P,
+]
+_lib.mcpu_paged_attention_forward_fp8.restype = ctypes.c_int
 _lib.mcpu_read_device_status.argtypes = [_P, _P, ctypes.POINTER(ctypes.c_int32)]
 _lib.mcpu_read_device_status.restype = ctypes.c_int
 _lib.mcpu_reset_device_status.argtypes = [_P, _P]
@@ -203,16 +212,10 @@ def mcpu_grow_block_tables(block_table, seq_lens, free_pages, free_count, status
     )
 
 
-def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, sliding_window,
-                                 softmax_scale, out, lse, workspace, flags=0, split_pages=0, stream=None,
-                                 phase_events=None, sinks=None):
-    """phase_events: optional list of NUM_PHASE_EVENTS torch.cuda.Event the
-    call records around its kernels (see mcpu_options in include/mcpu.h);
-    sinks: optional float32 device tensor [H_q] of attention-sink logits."""
-    d = dims(q, k_cache, block_table, seq_lens)
+def _options(num_q_heads, flags, split_pages, phase_events, sinks) -> Options:
     opts = Options(flags=int(flags), split_pages=int(split_pages), phase_events=None, sinks=None)
     if sinks is not None:
-        if sinks.dtype != torch.float32 or sinks.numel() != d.num_q_heads or not sinks.is_cuda:
+        if sinks.dtype != torch.float32 or sinks.numel() != num_q_heads or not sinks.is_cuda:
             raise ValueError("sinks must be a float32 CUDA tensor with one value per q head")
         opts.sinks = ctypes.c_void_p(sinks.data_ptr())
     if phase_events is not None:
@@ -222,6 +225,18 @@ def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, que
                              "before passing it")
         arr = (ctypes.c_void_p * NUM_PHASE_EVENTS)(*[ctypes.c_void_p(e.cuda_event) for e in phase_events])
         opts.phase_events = ctypes.cast(arr, ctypes.c_void_p)
+        opts._events = arr  # keep the array alive as long as the options
+    return opts
+
+
+def mcpu_paged_attention_forward(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, sliding_window,
+                                 softmax_scale, out, lse, workspace, flags=0, split_pages=0, stream=None,
+                                 phase_events=None, sinks=None):
+    """phase_events: optional list of NUM_PHASE_EVENTS torch.cuda.Event the
+    call records around its kernels (see mcpu_options in include/mcpu.h);
+    sinks: optional float32 device tensor [H_q] of attention-sink logits."""
+    d = dims(q, k_cache, block_table, seq_lens)
+    opts = _options(d.num_q_heads, flags, split_pages, phase_events, sinks)
     _check(
         _lib.mcpu_paged_attention_forward(
             _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc),
@@ -244,6 +259,45 @@ def mcpu_paged_attention_forward_noalloc(q, k_cache, v_cache, block_table, seq_l
             _stream(stream),
         ),
         "mcpu_paged_attention_forward_noalloc",
+    )
+
+
+def mcpu_kv_append_fp8(k_new, v_new, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc,
+                       status_word, stream=None):
+    """Quantizing KV append into fp8 pools: k8 uint8 [P, Hkv, 16, D], v8 uint8
+    [P, Hkv, D, 16] (each block transposed), scales float32 [P, Hkv, 16]."""
+    d = Dims(
+        num_seqs=int(seq_lens.shape[0]),
+        total_q=int(k_new.shape[0]),
+        max_pages_per_seq=int(block_table.shape[1]),
+        num_pages=int(k8.shape[0]),
+        num_q_heads=int(k8.shape[1]),
+        num_kv_heads=int(k8.shape[1]),
+        head_dim=int(k8.shape[3]),
+        page_size=int(k8.shape[2]),
+    )
+    _check(
+        _lib.mcpu_kv_append_fp8(_ptr(k_new), _ptr(v_new), _ptr(k8), _ptr(v8), _ptr(k_scale), _ptr(v_scale),
+                                _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc), ctypes.byref(d),
+                                _ptr(status_word), _stream(stream)),
+        "mcpu_kv_append_fp8",
+    )
+
+
+def mcpu_paged_attention_forward_fp8(q, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc,
+                                     sliding_window, softmax_scale, out, lse, workspace, flags=0, split_pages=0,
+                                     stream=None, phase_events=None, sinks=None):
+    """Decode-row attention over fp8 pools (layouts as mcpu_kv_append_fp8)."""
+    d = dims(q, k8, block_table, seq_lens)
+    opts = _options(d.num_q_heads, flags, split_pages, phase_events, sinks)
+    _check(
+        _lib.mcpu_paged_attention_forward_fp8(
+            _ptr(q), _ptr(k8), _ptr(v8), _ptr(k_scale), _ptr(v_scale), _ptr(block_table), _ptr(seq_lens),
+            _ptr(query_start_loc), int(sliding_window), float(softmax_scale), ctypes.byref(d), _ptr(out), _ptr(lse),
+            _ptr(workspace), int(workspace.numel() * workspace.element_size()), ctypes.byref(opts),
+            _stream(stream),
+        ),
+        "mcpu_paged_attention_forward_fp8",
     )
 
 

@@ -118,3 +118,99 @@ def assert_parity(got_out, got_lse, ref_out, ref_lse, what=""):
     assert rel <= OUT_REL, f"{what}: norm-relative err {rel:.3e}"
     assert lse_err <= LSE_ABS, f"{what}: lse abs err {lse_err:.3e}"
     return max_abs, rel, lse_err
+
+
+# ------------------------------------------------------------ fp8 pools
+
+
+def oracle_quantize_pool(k_bits, v_bits):
+    """fp8 pools (codes [P, Hkv, 16, D] uint8 both, scales [P, Hkv, 16]) of
+    whole bf16 pools, quantized by the oracle: every page is appended as one
+    16-token row."""
+    P, H, page, D = k_bits.shape
+    tok = lambda x: np.ascontiguousarray(np.asarray(x).transpose(0, 2, 1, 3).reshape(P * page, H, D))  # noqa: E731
+    z8 = np.zeros((P, H, page, D), np.uint8)
+    zs = np.zeros((P, H, page), np.float32)
+    bt = np.arange(P, dtype=np.int32)[:, None]
+    sl = np.full(P, page, np.int32)
+    qsl = (np.arange(P + 1, dtype=np.int32) * page)
+    return oracle.kv_append_fp8(tok(k_bits), tok(v_bits), z8, z8, zs, zs, bt, sl, qsl)
+
+
+def v_to_device_layout(v8):
+    """Oracle V codes [P, Hkv, 16, D] -> the ABI's transposed blocks [P, Hkv, D, 16]."""
+    return np.ascontiguousarray(np.asarray(v8).transpose(0, 1, 3, 2))
+
+
+class Fp8Run:
+    """A decode batch on fp8 pools: the prior context quantized by the oracle
+    and uploaded, then this step's rows appended on the device by
+    mcpu_kv_append_fp8 (checked bit for bit against the oracle's append)."""
+
+    def __init__(self, batch: W.Batch, layer: int = 0, device="cuda", garbage_slots=False):
+        self.batch = batch
+        self.layer = layer
+        h = W.host_inputs(batch, layer)
+        self.h = h
+        k8, v8, ks, vs = oracle_quantize_pool(h["k_cache"], h["v_cache"])
+        if garbage_slots:
+            # slots no row can see hold NaN codes and NaN scales
+            vis = np.zeros(ks.shape[0:1] + ks.shape[2:], bool)  # [P, 16]
+            bt, sl = h["block_table"], h["seq_lens"]
+            for r in range(len(sl)):
+                for j in range(int(sl[r])):
+                    vis[bt[r, j // 16], j % 16] = True
+            hide = ~vis
+            k8 = k8.copy(); v8 = v8.copy(); ks = ks.copy(); vs = vs.copy()
+            k8.transpose(0, 2, 1, 3)[hide] = 0x7F
+            v8.transpose(0, 2, 1, 3)[hide] = 0xFF
+            ks.transpose(0, 2, 1)[hide] = np.nan
+            vs.transpose(0, 2, 1)[hide] = np.nan
+        self.before = (k8, v8, ks, vs)
+        dev = torch.device(device)
+        lay = batch.layers[layer]
+        self.q = lay.q.to(dev)
+        self.k_new = lay.k_new.to(dev)
+        self.v_new = lay.v_new.to(dev)
+        self.k8 = torch.from_numpy(k8).to(dev)
+        self.v8 = torch.from_numpy(v_to_device_layout(v8)).to(dev)
+        self.ks = torch.from_numpy(ks).to(dev)
+        self.vs = torch.from_numpy(vs).to(dev)
+        pool = batch.pools[lay.pool]
+        self.bt = torch.from_numpy(pool.block_table).to(dev)
+        self.sl = torch.from_numpy(batch.seq_lens).to(dev)
+        self.qsl = torch.from_numpy(batch.query_start_loc).to(dev)
+        self.window = lay.sliding_window
+        self.dims = mcpu.dims(self.q, self.k8, self.bt, self.sl)
+        self.ws = mcpu.new_workspace(self.dims, dev)
+        self.out = torch.full_like(self.q, float("nan"))
+        self.lse = torch.full(self.q.shape[:2], float("nan"), dtype=torch.float32, device=dev)
+
+    def append(self):
+        mcpu.mcpu_kv_append_fp8(self.k_new, self.v_new, self.k8, self.v8, self.ks, self.vs, self.bt, self.sl,
+                                self.qsl, mcpu.status_word(self.ws))
+
+    def oracle_append(self):
+        h = self.h
+        return oracle.kv_append_fp8(h["k_new"], h["v_new"], *self.before, h["block_table"], h["seq_lens"],
+                                    h["query_start_loc"])
+
+    def forward(self, flags=0, split_pages=0, sinks=None):
+        sk = None if sinks is None else torch.from_numpy(np.asarray(sinks, np.float32)).to(self.q.device)
+        mcpu.mcpu_paged_attention_forward_fp8(self.q, self.k8, self.v8, self.ks, self.vs, self.bt, self.sl,
+                                              self.qsl, self.window, self.batch.softmax_scale, self.out, self.lse,
+                                              self.ws, flags=flags, split_pages=split_pages, sinks=sk)
+
+    def status(self):
+        return mcpu.mcpu_read_device_status(self.ws)
+
+    def header(self):
+        hd = self.ws[:32].view(torch.int32).cpu().numpy()
+        return dict(status=int(hd[0]), n_decode=int(hd[1]), n_cascade=int(hd[2]), n_append=int(hd[3]),
+                    n_merge=int(hd[4]), split_pages=int(hd[5]), n_parts=int(hd[6]))
+
+    def pools_host(self):
+        return (self.k8.cpu().numpy(), self.v8.cpu().numpy(), self.ks.cpu().numpy(), self.vs.cpu().numpy())
+
+    def out_host(self):
+        return self.out.float().cpu().numpy(), self.lse.cpu().numpy()
