@@ -297,18 +297,16 @@ class Stepper:
 
 
 def quantize_pools_fp8(batch: W.Batch, dev):
-    """fp8 copies of every pool, written by mcpu_kv_append_fp8 with every
-    page appended as one 16-token row (input preparation, untimed)."""
+    """An fp8 pool (uint8 [P, Hkv, 2176]) for every bf16 pool, written by
+    mcpu_kv_append_fp8 with every page appended as one 16-token row (input
+    preparation, untimed)."""
     from paper_2608_22167_gb300 import mcpu
 
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     pools = {}
     for key, pool in batch.pools.items():
         P, H, page, D = pool.k_cache.shape
-        k8 = torch.empty((P, H, page, D), dtype=torch.uint8, device=dev)
-        v8 = torch.empty((P, H, D, page), dtype=torch.uint8, device=dev)
-        ks = torch.empty((P, H, page), dtype=torch.float32, device=dev)
-        vs = torch.empty_like(ks)
+        kv8 = mcpu.new_fp8_pool(P, H, dev)
         chunk = 2048  # rows per call (the planner's row limit)
         for p0 in range(0, P, chunk):
             n = min(chunk, P - p0)
@@ -317,8 +315,8 @@ def quantize_pools_fp8(batch: W.Batch, dev):
             bt = torch.arange(p0, p0 + n, dtype=torch.int32, device=dev).view(n, 1)
             sl = torch.full((n,), page, dtype=torch.int32, device=dev)
             qsl = torch.arange(0, (n + 1) * page, page, dtype=torch.int32, device=dev)
-            mcpu.mcpu_kv_append_fp8(kn, vn, k8, v8, ks, vs, bt, sl, qsl, status)
-        pools[key] = (k8, v8, ks, vs)
+            mcpu.mcpu_kv_append_fp8(kn, vn, kv8, bt, sl, qsl, status)
+        pools[key] = kv8
     torch.cuda.synchronize()
     if int(status.item()) != 0:
         raise RuntimeError(f"fp8 pool quantization: device status {int(status.item())}")
@@ -338,14 +336,13 @@ class Fp8Stepper(Stepper):
     def layer_call(self, i, q=None, k_new=None, v_new=None, out=None, lse=None, events=None):
         m = self.mcpu
         lay = self.layers[i]
-        k8, v8, ks, vs = self.pools8[lay.pool]
+        kv8 = self.pools8[lay.pool]
         bt = self.bts[lay.pool]
         m.mcpu_kv_append_fp8(lay.k_new if k_new is None else k_new, lay.v_new if v_new is None else v_new,
-                             k8, v8, ks, vs, bt, self.sl, self.qsl, m.status_word(self.ws))
-        m.mcpu_paged_attention_forward_fp8(lay.q if q is None else q, k8, v8, ks, vs, bt, self.sl, self.qsl,
-                                           lay.sliding_window, self.batch.softmax_scale,
-                                           self.out if out is None else out, self.lse if lse is None else lse,
-                                           self.ws, phase_events=events)
+                             kv8, bt, self.sl, self.qsl, m.status_word(self.ws))
+        m.mcpu_paged_attention_forward_fp8(lay.q if q is None else q, kv8, bt, self.sl, self.qsl, lay.sliding_window,
+                                           self.batch.softmax_scale, self.out if out is None else out,
+                                           self.lse if lse is None else lse, self.ws, phase_events=events)
 
 
 def make_batch(name, dev, rank):

@@ -244,35 +244,38 @@ mcpu_status mcpu_grow_block_tables(int32_t* block_table, const int32_t* seq_lens
  * K[j][d] = value(code) * scale. One scale per row rather than per page, so
  * that a page can fill one token at a time without requantizing.
  *
- * Layouts (device memory, 16-byte aligned):
- *   k8       [num_pages, H_kv, 16, D] uint8  codes, one 64-byte row per key
- *   v8       [num_pages, H_kv, D, 16] uint8  codes, each (page, kv head)
- *            block TRANSPOSED: v8[page][h][d][slot]
- *   k_scale, v_scale [num_pages, H_kv, 16] float
- * Slots of a page that no row has written may hold anything: the kernels
- * mask them (their codes become finite numbers that are multiplied by 0).
+ * Layout: one pool `kv8` of num_pages * H_kv blocks of 2176 bytes, block
+ * (page, h) at byte offset (page * H_kv + h) * 2176 (16-byte aligned base):
+ *   bytes    0..1023  K codes, uint8 [16 slots][D]
+ *   bytes 1024..2047  V codes, uint8 [D][16 slots]   (transposed)
+ *   bytes 2048..2111  K scales, float [16 slots]
+ *   bytes 2112..2175  V scales, float [16 slots]
+ * so that one copy brings a page's K, V and scales (a 16-token page takes
+ * 2176 bytes per kv head instead of 4096 in bf16). Slots that no row has
+ * written may hold anything: the kernels mask them.
  *
  * mcpu_kv_append_fp8: as mcpu_kv_append (same placement, lengths and error
- * bits), quantizing each new row as above; k_new, v_new stay bf16.
+ * bits), quantizing each new K and V row as above; k_new, v_new stay bf16.
  */
-mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
-                               float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
-                               const int32_t* query_start_loc, const mcpu_dims* dims, int32_t* status_word,
-                               mcpu_stream_t stream);
+mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* kv8, const int32_t* block_table,
+                               const int32_t* seq_lens, const int32_t* query_start_loc, const mcpu_dims* dims,
+                               int32_t* status_word, mcpu_stream_t stream);
 
 /*
  * mcpu_paged_attention_forward over fp8 pages, for decode rows (L_r = 1 or
  * 0): same arguments, results and options as mcpu_paged_attention_forward
  * (split-KV, cascade pass over shared prompt pages, sliding window, sinks,
- * phase events, graph capture), with the pools replaced by the four fp8
- * arrays. dims->num_pages counts pages of k8 (and v8). A batch with
- * total_q > num_seqs (some row appends) returns MCPU_ERR_UNSUPPORTED
- * without launching; an append row found on the device is skipped and
- * reported as MCPU_ERR_UNSUPPORTED_ROW. MCPU_FLAG_MMA_SYNC_APPEND is not
- * accepted; every kernel runs on `stream`.
+ * phase events, graph capture), with the two bf16 pools replaced by kv8.
+ * dims->num_pages counts pages of kv8. The products run on the fp8 tensor
+ * cores: q is carried as three e4m3 pieces (exact to about 2^-12 of a query
+ * vector's largest entry) and the softmax weights times the V scales as two
+ * (fp16 rounded, then to about 2^-8 relative), accumulation in fp32.
+ * A batch with total_q > num_seqs (some row appends) returns
+ * MCPU_ERR_UNSUPPORTED without launching; an append row found on the device
+ * is skipped and reported as MCPU_ERR_UNSUPPORTED_ROW. MCPU_FLAG_MMA_SYNC_APPEND
+ * is not accepted; every kernel runs on `stream`.
  */
-mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* k8, const void* v8, const float* k_scale,
-                                             const float* v_scale, const int32_t* block_table,
+mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, const int32_t* block_table,
                                              const int32_t* seq_lens, const int32_t* query_start_loc,
                                              int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
                                              void* out, float* lse, void* workspace, size_t workspace_bytes,

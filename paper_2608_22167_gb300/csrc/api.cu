@@ -37,12 +37,11 @@ cudaError_t launch_kv_append(const void* k_new, const void* v_new, void* k_cache
                              const int32_t* block_table, const int32_t* seq_lens, const int32_t* qsl,
                              int32_t* status, int32_t num_seqs, int32_t total_q, int32_t max_pages,
                              int32_t num_pages, int32_t num_kv_heads, cudaStream_t stream);
-cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
-                                 float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
-                                 const int32_t* qsl, int32_t* status, int32_t num_seqs, int32_t total_q,
-                                 int32_t max_pages, int32_t num_pages, int32_t num_kv_heads, cudaStream_t stream);
-cudaError_t launch_decode_fp8(const void* k8, const void* v8, const float* k_scale, const float* v_scale,
-                              const AttnParams& p, int grid, bool cascade, cudaStream_t stream);
+cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* kv8, const int32_t* block_table,
+                                 const int32_t* seq_lens, const int32_t* qsl, int32_t* status, int32_t num_seqs,
+                                 int32_t total_q, int32_t max_pages, int32_t num_pages, int32_t num_kv_heads,
+                                 cudaStream_t stream);
+cudaError_t launch_decode_fp8(const void* kv8, const AttnParams& p, int grid, bool cascade, cudaStream_t stream);
 cudaError_t prepare_fp8_kernels(int* bpsm_decode, int* bpsm_cascade);
 }  // namespace mcpu
 
@@ -366,32 +365,27 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   return from_cuda(e);
 }
 
-mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
-                               float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
-                               const int32_t* query_start_loc, const mcpu_dims* dims, int32_t* status_word,
-                               mcpu_stream_t stream) {
+mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* kv8, const int32_t* block_table,
+                               const int32_t* seq_lens, const int32_t* query_start_loc, const mcpu_dims* dims,
+                               int32_t* status_word, mcpu_stream_t stream) {
   mcpu_status st = check_dims(dims);
   if (st != MCPU_OK) return st;
   if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
-  if (!k_new || !v_new || !k8 || !v8 || !k_scale || !v_scale || !block_table || !seq_lens || !query_start_loc ||
-      !status_word)
+  if (!k_new || !v_new || !kv8 || !block_table || !seq_lens || !query_start_loc || !status_word)
     return MCPU_ERR_INVALID_ARG;
-  if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k8, 16) || !aligned(v8, 16) || !aligned(k_scale, 16) ||
-      !aligned(v_scale, 16) || !aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(query_start_loc, 4) ||
-      !aligned(status_word, 4))
+  if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(kv8, 16) || !aligned(block_table, 4) ||
+      !aligned(seq_lens, 4) || !aligned(query_start_loc, 4) || !aligned(status_word, 4))
     return MCPU_ERR_INVALID_ARG;
   if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
   DeviceState* dev = nullptr;
   st = device_state(&dev);
   if (st != MCPU_OK) return st;
-  return from_cuda(launch_kv_append_fp8(k_new, v_new, k8, v8, k_scale, v_scale, block_table, seq_lens,
-                                        query_start_loc, status_word, dims->num_seqs, dims->total_q,
-                                        dims->max_pages_per_seq, dims->num_pages, dims->num_kv_heads,
-                                        reinterpret_cast<cudaStream_t>(stream)));
+  return from_cuda(launch_kv_append_fp8(k_new, v_new, kv8, block_table, seq_lens, query_start_loc, status_word,
+                                        dims->num_seqs, dims->total_q, dims->max_pages_per_seq, dims->num_pages,
+                                        dims->num_kv_heads, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* k8, const void* v8, const float* k_scale,
-                                             const float* v_scale, const int32_t* block_table,
+mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, const int32_t* block_table,
                                              const int32_t* seq_lens, const int32_t* query_start_loc,
                                              int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
                                              void* out, float* lse, void* workspace, size_t workspace_bytes,
@@ -405,11 +399,9 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* k8, cons
   if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_OK;
   // decode rows only: more query tokens than rows means some row appends
   if (dims->total_q > dims->num_seqs) return MCPU_ERR_UNSUPPORTED;
-  if (!q || !k8 || !v8 || !k_scale || !v_scale || !block_table || !seq_lens || !query_start_loc || !out || !lse)
-    return MCPU_ERR_INVALID_ARG;
-  if (!aligned(q, 16) || !aligned(k8, 16) || !aligned(v8, 16) || !aligned(k_scale, 16) || !aligned(v_scale, 16) ||
-      !aligned(out, 16) || !aligned(lse, 4) || !aligned(block_table, 4) || !aligned(seq_lens, 4) ||
-      !aligned(query_start_loc, 4))
+  if (!q || !kv8 || !block_table || !seq_lens || !query_start_loc || !out || !lse) return MCPU_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(kv8, 16) || !aligned(out, 16) || !aligned(lse, 4) || !aligned(block_table, 4) ||
+      !aligned(seq_lens, 4) || !aligned(query_start_loc, 4))
     return MCPU_ERR_INVALID_ARG;
   if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
   if (opts && opts->split_pages < 0) return MCPU_ERR_INVALID_ARG;
@@ -462,10 +454,10 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* k8, cons
   cudaError_t e = mark(0);
   if (e == cudaSuccess) e = launch_plan(p, s);
   if (e == cudaSuccess) e = mark(1);
-  if (e == cudaSuccess) e = launch_decode_fp8(k8, v8, k_scale, v_scale, p, dev->sms * dev->bpsm_fp8, false, s);
+  if (e == cudaSuccess) e = launch_decode_fp8(kv8, p, dev->sms * dev->bpsm_fp8, false, s);
   if (e == cudaSuccess) e = mark(2);
   if (e == cudaSuccess && cascade)
-    e = launch_decode_fp8(k8, v8, k_scale, v_scale, p, dev->sms * dev->bpsm_fp8_cascade, true, s);
+    e = launch_decode_fp8(kv8, p, dev->sms * dev->bpsm_fp8_cascade, true, s);
   if (e == cudaSuccess) e = mark(3);
   if (e == cudaSuccess) e = mark(4);
   if (e == cudaSuccess) {

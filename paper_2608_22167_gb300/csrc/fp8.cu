@@ -1,33 +1,37 @@
 // fp8 (e4m3) KV pages: the quantizing KV append and the split-KV decode /
 // cascade kernel that reads them (a storage variant; the paper keeps bf16).
 //
-// Storage, per (page, kv head) block:
-//   k8  [16 keys][64 dims]  e4m3 codes, row-major (1 KiB)
-//   v8  [64 dims][16 keys]  e4m3 codes, TRANSPOSED (1 KiB)
-//   k_scale, v_scale [16]   float, one scale per (token, kv head) row
-// Each new row x (64 bf16) is stored as a = max|x_i|, scale = a / 448 and
-// code_i = e4m3(x_i * (448 / a)) (round to nearest even, saturating), in
+// Storage: one 2176-byte block per (page, kv head), blocks ordered
+// [page][kv head]:
+//   bytes    0..1023  K codes [16 keys][64 dims]  (row-major)
+//   bytes 1024..2047  V codes [64 dims][16 keys]  (transposed)
+//   bytes 2048..2111  K scales [16] float
+//   bytes 2112..2175  V scales [16] float
+// Each new row x (64 bf16 values) is stored as a = max|x_i|, scale = a / 448
+// and code_i = e4m3(x_i * (448 / a)) (round to nearest even, saturating), in
 // float arithmetic; an all-zero row stores zeros. A key is code * scale.
 //
-// Decode over fp8 pages follows the bf16 kernel (one warp per work item,
-// a per-warp ring of pages, m16n8k16 tensor-core tiles, online softmax,
-// partials merged by log-sum-exp) with these differences:
-//   - a page's 2 KiB of codes and 128 B of scales arrive by four untiled
-//     bulk copies (no tensor map), 2176 bytes per (page, kv head);
-//   - codes become fp16 operands by integer ops: an e4m3 code c placed in
-//     the high byte of a 16-bit lane gives ((c & 0x7f) << 7) | sign, the
-//     fp16 whose value is exactly value(c) * 2^-8 (subnormals included), so
-//     both products run as f16 x f16 -> f32;
-//   - q enters as fp16 times a power of two per query vector (its largest
-//     entry lands in [2^14, 2^15)); the key scale, that power of two and
-//     the softmax scale multiply each score in fp32;
-//   - P . V takes P' = p * v_scale * 2^8 * 2^F in fp16, F a per-item power
-//     of two that only decreases (the page's largest v_scale sets it, so P'
-//     stays below 2^15); the accumulator is rescaled when F drops and
-//     divided by 2^F at the end.
-// Which dims/keys meet in one MMA k-slot is a permutation chosen so that
-// every operand comes from a 32- or 128-bit shared-memory load: row 2r and
-// 2r + 1 of the K block and word c (keys 4c..4c+3) of the transposed V rows.
+// Decode over fp8 pages follows the bf16 kernel (one warp per work item, a
+// per-warp ring of pages filled by one bulk copy each, online softmax in
+// fp32, partials merged by log-sum-exp) but multiplies on the fp8 tensor
+// cores (mma m16n8k32, e4m3 x e4m3 -> f32), so the codes go from shared
+// memory into the MMAs as they are:
+//   - S = K q: q (bf16) times a power of two per query vector (largest
+//     entry in [2^7, 2^8)) is split into three e4m3 pieces hi + mid + lo,
+//     exact to ~2^-12 of the largest entry; the hi and mid pieces share one
+//     MMA through a duplicated K operand, lo pieces take two more (6 per
+//     page). Each score is then scaled by its key's scale, the power of two
+//     and the softmax scale;
+//   - O += P' V: P' = p * v_scale * 2^F in fp16 (F a per-item power of two
+//     that only decreases, so that P' < 2^8) is split into e4m3 hi + lo, the
+//     two pieces sit in the two halves of the MMA's k range beside a
+//     duplicated V operand (4 MMAs per page). The accumulator is rescaled
+//     when F drops and divided by 2^F at the end.
+// Which keys meet in which MMA row/slot is a permutation chosen so that the
+// score fragment transposes into the P' operand with movmatrix: M row r of
+// the score tile is key 4(r/2) + (r%2), row r + 8 is that key + 2. V codes of
+// keys a row cannot see are zeroed in registers (unwritten slots may hold
+// any byte, e4m3 NaN included); a page outside the pool is skipped.
 #include <cuda_fp16.h>
 
 #include "common.cuh"
@@ -36,30 +40,63 @@ namespace mcpu {
 
 constexpr int kF8Warps = 4;
 constexpr int kF8Stages = 8;
-constexpr int kF8Block = kPage * kHeadDim;                      // codes of one block: 1 KiB
-constexpr int kF8ScaleBytes = kPage * 4;                        // 64
-constexpr int kF8StageBytes = 2 * kF8Block + 2 * kF8ScaleBytes;  // 2176
-constexpr int kF8RingBytes = kF8Stages * kF8StageBytes;
-
-struct F8Pools {
-  const uint8_t* k8;
-  const uint8_t* v8;
-  const float* k_scale;
-  const float* v_scale;
-};
+constexpr int kF8Codes = kPage * kHeadDim;  // 1024 codes per (page, kv head) for K, and for V
+constexpr int kF8VOff = kF8Codes;
+constexpr int kF8KsOff = 2 * kF8Codes;
+constexpr int kF8VsOff = 2 * kF8Codes + kPage * 4;
+constexpr int kF8BlockBytes = 2 * kF8Codes + 2 * kPage * 4;  // 2176
+constexpr int kF8RingBytes = kF8Stages * kF8BlockBytes;
 
 size_t decode_fp8_smem_bytes() {
   return 128 /* alignment slack */ + (size_t)kF8Warps * kF8RingBytes + (size_t)kF8Warps * kF8Stages * 8;
 }
 
-// Two e4m3 codes in bits 8..15 and 24..31 of y -> f16x2 of value(code) * 2^-8.
-__device__ __forceinline__ uint32_t e4m3_pair_to_f16x2(uint32_t y) {
-  return ((y >> 1) & 0x3F803F80u) | (y & 0x80008000u);
+// D = A(16x32, row) * B(32x8, col) + D, e4m3 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_e4m3_16832(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
+// e4m3 codes of x0 (low byte) and x1 (high byte): nearest, ties to even,
+// saturating at +-448.
+__device__ __forceinline__ uint32_t e4m3x2(float x0, float x1) {
+  uint16_t d;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(d) : "f"(x1), "f"(x0));
+  return d;
+}
+// the same from an f16 pair (low half -> low byte)
+__device__ __forceinline__ uint32_t e4m3x2_from_f16x2(uint32_t h) {
+  uint16_t d;
+  asm("cvt.rn.satfinite.e4m3x2.f16x2 %0, %1;" : "=h"(d) : "r"(h));
+  return d;
+}
+// exact f16 pair of two codes (low byte -> low half)
+__device__ __forceinline__ uint32_t f16x2_from_e4m3x2(uint32_t c) {
+  uint32_t h;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h) : "h"((uint16_t)c));
+  return h;
+}
 __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
   __half2 v = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ uint32_t hsub2_u32(uint32_t a, uint32_t b) {
+  __half2 r = __hsub2(*reinterpret_cast<__half2*>(&a), *reinterpret_cast<__half2*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+  return d;
+}
+// value of each code of a pair, as floats
+__device__ __forceinline__ float2 e4m3x2_value(uint32_t c) {
+  const uint32_t h = f16x2_from_e4m3x2(c);
+  return __half22float2(*reinterpret_cast<const __half2*>(&h));
 }
 
 // 2^e as a float for -126 <= e <= 127
@@ -68,11 +105,21 @@ __device__ __forceinline__ float exp2i(int e) { return __uint_as_float((uint32_t
 // floor(log2(x)) of a positive finite float (subnormals give -127)
 __device__ __forceinline__ int ilog2f(float x) { return (int)((__float_as_uint(x) >> 23) & 0xFF) - 127; }
 
+// Byte mask of the keys 4c..4c+3 of a page that lie in [lo, hi).
+__device__ __forceinline__ uint32_t key_byte_mask(int c, int lo, int hi) {
+  uint32_t m = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) m |= (4 * c + i >= lo && 4 * c + i < hi) ? (0xFFu << (8 * i)) : 0u;
+  return m;
+}
+
 template <int NT>
-__global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools pools, const AttnParams p) {
+__global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t* __restrict__ kv8,
+                                                                   const AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
+  const int key_a = 4 * (r >> 1) + (r & 1), key_b = key_a + 2;  // keys of M rows r and r + 8
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 127u) & ~127u;
   const uint32_t ring = base + warp * kF8RingBytes;
@@ -127,10 +174,11 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
     }
     const int* bt_row = p.block_table + (size_t)row * p.max_pages;
 
-    // Query vector r (+ 8 nt) as the B operand: this lane holds its dims
-    // 16c .. 16c + 15 times 2^eq; k-slot 2c + e of step kk is dim
-    // 16c + 4kk + 2e, k-slot 2c + 8 + e is dim 16c + 4kk + 1 + 2e.
-    uint32_t qb[NT][4][2];
+    // Query vector r (+ 8 nt) as B operands: this lane holds its dims
+    // 16c .. 16c + 15 as e4m3 pieces of q * 2^eq. Step s of the hi/mid MMAs
+    // takes dims 16c + 4s .. + 3 (hi in k-slots 0..15, mid in 16..31); the
+    // two lo MMAs take dims 16c + 8t .. + 3 and 16c + 8t + 4 .. + 3.
+    uint32_t q_hi[NT][4], q_mid[NT][4], q_lo[NT][4];
     float qm[NT][2];  // score factor of query vectors 2c and 2c + 1
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
@@ -161,15 +209,30 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
       for (int i = 0; i < 16; ++i) mx = fmaxf(mx, fabsf(x[i]));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      int eq = mx > 0.f ? 14 - ilog2f(mx) : 0;
+      int eq = mx > 0.f ? 7 - ilog2f(mx) : 0;
       eq = min(max(eq, -126), 126);
       const float up = exp2i(eq);
-      const float my_qm = exp2i(-eq) * 256.f * p.scale_log2;
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        qb[nt][kk][0] = pack_f16x2(x[4 * kk] * up, x[4 * kk + 2] * up);
-        qb[nt][kk][1] = pack_f16x2(x[4 * kk + 1] * up, x[4 * kk + 3] * up);
+      for (int j = 0; j < 4; ++j) {  // word j: dims 16c + 4j .. + 3
+        uint32_t h = 0, m = 0, l = 0;
+#pragma unroll
+        for (int i = 0; i < 4; i += 2) {
+          const float a0 = x[4 * j + i] * up, a1 = x[4 * j + i + 1] * up;
+          const uint32_t ch = e4m3x2(a0, a1);
+          const float2 vh = e4m3x2_value(ch);
+          const float r0 = a0 - vh.x, r1 = a1 - vh.y;  // exact
+          const uint32_t cm = e4m3x2(r0, r1);
+          const float2 vm = e4m3x2_value(cm);
+          const uint32_t cl = e4m3x2(r0 - vm.x, r1 - vm.y);
+          h |= ch << (8 * i);
+          m |= cm << (8 * i);
+          l |= cl << (8 * i);
+        }
+        q_hi[nt][j] = h;
+        q_mid[nt][j] = m;
+        q_lo[nt][j] = l;
       }
+      const float my_qm = exp2i(-eq) * p.scale_log2;
       qm[nt][0] = __shfl_sync(0xffffffffu, my_qm, (2 * c) * 4);
       qm[nt][1] = __shfl_sync(0xffffffffu, my_qm, (2 * c + 1) * 4);
     }
@@ -177,7 +240,7 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
     // Page ids: lane i caches the id of page (chunk + i); lane 0 issues.
     const int n = pe - pb;
     int chunk_base = -32, pid_reg = 0;
-    uint32_t bad_stages = 0;  // stages holding an invalid page (warp-uniform)
+    uint32_t bad_stages = 0;  // stages holding no page (warp-uniform)
     auto page_id = [&](int k) -> int {
       const int cb = k & ~31;
       if (cb != chunk_base) {
@@ -202,15 +265,11 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
       if (lane == 0) {
         const uint32_t bar = bars + 8 * s;
         if (pid < 0) {
-          mbar_arrive(bar);  // nothing to copy: the page's keys are masked
+          mbar_arrive(bar);  // nothing to copy: the page is skipped
         } else {
-          const size_t blk = (size_t)pid * Hkv + kvh;
-          const uint32_t dst = ring + s * kF8StageBytes;
-          mbar_arrive_expect_tx(bar, kF8StageBytes);
-          bulk_load(dst, pools.k8 + blk * kF8Block, kF8Block, bar, pol);
-          bulk_load(dst + kF8Block, pools.v8 + blk * kF8Block, kF8Block, bar, pol);
-          bulk_load(dst + 2 * kF8Block, pools.k_scale + blk * kPage, kF8ScaleBytes, bar, pol);
-          bulk_load(dst + 2 * kF8Block + kF8ScaleBytes, pools.v_scale + blk * kPage, kF8ScaleBytes, bar, pol);
+          mbar_arrive_expect_tx(bar, kF8BlockBytes);
+          bulk_load(ring + s * kF8BlockBytes, kv8 + ((size_t)pid * Hkv + kvh) * kF8BlockBytes, kF8BlockBytes, bar,
+                    pol);
         }
       }
     };
@@ -227,7 +286,7 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
     }
-    int F = 120;  // P' = p * v_scale * 2^8 * 2^F; acc is held in units of 2^F
+    int F = 120;  // P' = p * v_scale * 2^F; acc is held in units of 2^F
 
     bool timed_out = false;
     for (int k = 0; k < n; ++k) {
@@ -238,93 +297,106 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
         timed_out = true;
         break;
       }
-      const uint8_t* st = ring_ptr + s * kF8StageBytes;
-      const uint4 KA = *reinterpret_cast<const uint4*>(st + (2 * r) * kHeadDim + 16 * c);
-      const uint4 KB = *reinterpret_cast<const uint4*>(st + (2 * r + 1) * kHeadDim + 16 * c);
-      const float2 ks = *reinterpret_cast<const float2*>(st + 2 * kF8Block + 8 * r);
-      const float2 vs = *reinterpret_cast<const float2*>(st + 2 * kF8Block + kF8ScaleBytes + 8 * r);
+      if (!((bad_stages >> s) & 1u)) {
+        const uint8_t* st = ring_ptr + s * kF8BlockBytes;
+        const uint4 KA = *reinterpret_cast<const uint4*>(st + key_a * kHeadDim + 16 * c);
+        const uint4 KB = *reinterpret_cast<const uint4*>(st + key_b * kHeadDim + 16 * c);
+        const float* ksp = reinterpret_cast<const float*>(st + kF8KsOff);
+        const float* vsp = reinterpret_cast<const float*>(st + kF8VsOff);
+        const float ks0 = ksp[key_a], ks1 = ksp[key_b], vs0 = vsp[key_a], vs1 = vsp[key_b];
 
-      // S^T[16 keys x 8*NT query vectors]: M row r is key 2r, row r + 8 key 2r + 1
-      float cc[NT][4];
+        // S^T[16 keys x 8*NT query vectors] in units of q * 2^eq * K codes
+        float cc[NT][4];
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) cc[nt][0] = cc[nt][1] = cc[nt][2] = cc[nt][3] = 0.f;
-      {
-        const uint32_t wa[4] = {KA.x, KA.y, KA.z, KA.w}, wb[4] = {KB.x, KB.y, KB.z, KB.w};
+        for (int nt = 0; nt < NT; ++nt) cc[nt][0] = cc[nt][1] = cc[nt][2] = cc[nt][3] = 0.f;
+        {
+          const uint32_t wa[4] = {KA.x, KA.y, KA.z, KA.w}, wb[4] = {KB.x, KB.y, KB.z, KB.w};
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const uint32_t a0 = e4m3_pair_to_f16x2(wa[kk] << 8), a1 = e4m3_pair_to_f16x2(wb[kk] << 8);
-          const uint32_t a2 = e4m3_pair_to_f16x2(wa[kk]), a3 = e4m3_pair_to_f16x2(wb[kk]);
+          for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) mma_f16_16816(cc[nt], a0, a1, a2, a3, qb[nt][kk][0], qb[nt][kk][1]);
+            for (int j = 0; j < 4; ++j) mma_e4m3_16832(cc[nt], wa[j], wb[j], wa[j], wb[j], q_hi[nt][j], q_mid[nt][j]);
+#pragma unroll
+            for (int t = 0; t < 2; ++t)
+              mma_e4m3_16832(cc[nt], wa[2 * t], wb[2 * t], wa[2 * t + 1], wb[2 * t + 1], q_lo[nt][2 * t],
+                             q_lo[nt][2 * t + 1]);
+          }
         }
-      }
 
-      // keys outside [first_key, seq_len) or on an invalid page are masked
-      const int j0 = (pb + k) * kPage + 2 * r;
-      const bool page_ok = ((bad_stages >> s) & 1u) == 0;
-      bool v0 = page_ok, v1 = page_ok;
-      if (NT == 1) {
-        v0 = v0 && j0 >= first_key && j0 < seq_len;
-        v1 = v1 && (j0 + 1) >= first_key && (j0 + 1) < seq_len;
-      }
-      // the page's power of two for P' (F only decreases)
-      const float u0 = v0 ? vs.x * 256.f : 0.f, u1 = v1 ? vs.y * 256.f : 0.f;
-      float umax = fmaxf(u0, u1);
-      umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 4));
-      umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 8));
-      umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 16));
-      int F_new = F;
-      if (umax > 0.f) F_new = min(F, max(14 - ilog2f(umax), -120));
-      const float dF = F_new < F ? (F_new - F >= -126 ? exp2i(F_new - F) : 0.f) : 1.f;
-      F = F_new;
-      const float pf = exp2i(F);
-      const float w0 = u0 * pf, w1 = u1 * pf;
-
-      uint32_t pb0[NT], pb1[NT];
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        const float s00 = v0 ? cc[nt][0] * ks.x * qm[nt][0] : -INFINITY;
-        const float s01 = v0 ? cc[nt][1] * ks.x * qm[nt][1] : -INFINITY;
-        const float s10 = v1 ? cc[nt][2] * ks.y * qm[nt][0] : -INFINITY;
-        const float s11 = v1 ? cc[nt][3] * ks.y * qm[nt][1] : -INFINITY;
-        float mx0 = fmaxf(s00, s10), mx1 = fmaxf(s01, s11);
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-          mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-          mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+        // visible keys of this page: [klo, khi)
+        const int pk = (pb + k) * kPage;
+        int klo = 0, khi = kPage;
+        if (NT == 1) {
+          klo = max(first_key - pk, 0);
+          khi = min(seq_len - pk, kPage);
         }
-        const float mn0 = fmaxf(m_run[nt][0], mx0), mn1 = fmaxf(m_run[nt][1], mx1);
-        const float mu0 = mn0 == -INFINITY ? 0.f : mn0;
-        const float mu1 = mn1 == -INFINITY ? 0.f : mn1;
-        const float al0 = fast_exp2(m_run[nt][0] - mu0), al1 = fast_exp2(m_run[nt][1] - mu1);
-        const float p00 = fast_exp2(s00 - mu0), p10 = fast_exp2(s10 - mu0);
-        const float p01 = fast_exp2(s01 - mu1), p11 = fast_exp2(s11 - mu1);
-        l_run[nt][0] = l_run[nt][0] * al0 + p00 + p10;
-        l_run[nt][1] = l_run[nt][1] * al1 + p01 + p11;
-        m_run[nt][0] = mn0;
-        m_run[nt][1] = mn1;
-        const float ac0 = al0 * dF, ac1 = al1 * dF;
+        const bool v0 = key_a >= klo && key_a < khi, v1 = key_b >= klo && key_b < khi;
+        // the page's power of two for P' (F only decreases)
+        const float u0 = v0 ? vs0 : 0.f, u1 = v1 ? vs1 : 0.f;
+        float umax = fmaxf(u0, u1);
+        umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 4));
+        umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 8));
+        umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 16));
+        int F_new = F;
+        if (umax > 0.f) F_new = min(F, max(7 - ilog2f(umax), -120));
+        const float dF = F_new < F ? (F_new - F >= -126 ? exp2i(F_new - F) : 0.f) : 1.f;
+        F = F_new;
+        const float pf = exp2i(F);
+        const float w0 = u0 * pf, w1 = u1 * pf;
+
+        uint32_t pv_hi[NT], pv_lo[NT];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          const float s00 = v0 ? cc[nt][0] * ks0 * qm[nt][0] : -INFINITY;
+          const float s01 = v0 ? cc[nt][1] * ks0 * qm[nt][1] : -INFINITY;
+          const float s10 = v1 ? cc[nt][2] * ks1 * qm[nt][0] : -INFINITY;
+          const float s11 = v1 ? cc[nt][3] * ks1 * qm[nt][1] : -INFINITY;
+          float mx0 = fmaxf(s00, s10), mx1 = fmaxf(s01, s11);
+#pragma unroll
+          for (int o = 4; o < 32; o <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+          }
+          const float mn0 = fmaxf(m_run[nt][0], mx0), mn1 = fmaxf(m_run[nt][1], mx1);
+          const float mu0 = mn0 == -INFINITY ? 0.f : mn0;
+          const float mu1 = mn1 == -INFINITY ? 0.f : mn1;
+          const float al0 = fast_exp2(m_run[nt][0] - mu0), al1 = fast_exp2(m_run[nt][1] - mu1);
+          const float p00 = fast_exp2(s00 - mu0), p10 = fast_exp2(s10 - mu0);
+          const float p01 = fast_exp2(s01 - mu1), p11 = fast_exp2(s11 - mu1);
+          l_run[nt][0] = l_run[nt][0] * al0 + p00 + p10;
+          l_run[nt][1] = l_run[nt][1] * al1 + p01 + p11;
+          m_run[nt][0] = mn0;
+          m_run[nt][1] = mn1;
+          const float ac0 = al0 * dF, ac1 = al1 * dF;
+#pragma unroll
+          for (int mt = 0; mt < 4; ++mt) {
+            acc[mt][nt][0] *= ac0;
+            acc[mt][nt][1] *= ac1;
+            acc[mt][nt][2] *= ac0;
+            acc[mt][nt][3] *= ac1;
+          }
+          // P' in fp16, split into e4m3 hi + lo; each key's (hi, lo) codes
+          // form one 16-bit element for the transpose
+          const uint32_t fa = pack_f16x2(p00 * w0, p01 * w0), fb = pack_f16x2(p10 * w1, p11 * w1);
+          const uint32_t ha = e4m3x2_from_f16x2(fa), hb = e4m3x2_from_f16x2(fb);
+          const uint32_t la = e4m3x2_from_f16x2(hsub2_u32(fa, f16x2_from_e4m3x2(ha)));
+          const uint32_t lb = e4m3x2_from_f16x2(hsub2_u32(fb, f16x2_from_e4m3x2(hb)));
+          const uint32_t t0 = movmatrix_trans(prmt(ha, la, 0x5140u));  // keys 4c, 4c + 1 of column r
+          const uint32_t t1 = movmatrix_trans(prmt(hb, lb, 0x5140u));  // keys 4c + 2, 4c + 3
+          pv_hi[nt] = prmt(t0, t1, 0x6420u);
+          pv_lo[nt] = prmt(t0, t1, 0x7531u);
+        }
+
+        // O^T[64 dims x 8*NT] += V^T P'^T: k-slots 0..15 carry the hi piece,
+        // 16..31 the lo piece, both against the same V codes
+        const uint32_t vmask = (klo > 0 || khi < kPage) ? key_byte_mask(c, klo, khi) : 0xFFFFFFFFu;
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
-          acc[mt][nt][0] *= ac0;
-          acc[mt][nt][1] *= ac1;
-          acc[mt][nt][2] *= ac0;
-          acc[mt][nt][3] *= ac1;
+          const uint32_t x0 = *reinterpret_cast<const uint32_t*>(st + kF8VOff + (16 * mt + r) * kPage + 4 * c) & vmask;
+          const uint32_t x1 =
+              *reinterpret_cast<const uint32_t*>(st + kF8VOff + (16 * mt + r + 8) * kPage + 4 * c) & vmask;
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) mma_e4m3_16832(acc[mt][nt], x0, x1, x0, x1, pv_hi[nt], pv_lo[nt]);
         }
-        pb0[nt] = movmatrix_trans(pack_f16x2(p00 * w0, p01 * w0));
-        pb1[nt] = movmatrix_trans(pack_f16x2(p10 * w1, p11 * w1));
-      }
-
-      // O^T[64 dims x 8*NT] += V^T P'^T: k-slot 2c + e is key 4c + 2e,
-      // k-slot 2c + 8 + e is key 4c + 1 + 2e (word c of a transposed V row)
-#pragma unroll
-      for (int mt = 0; mt < 4; ++mt) {
-        const uint32_t x0 = *reinterpret_cast<const uint32_t*>(st + kF8Block + (16 * mt + r) * kPage + 4 * c);
-        const uint32_t x1 = *reinterpret_cast<const uint32_t*>(st + kF8Block + (16 * mt + r + 8) * kPage + 4 * c);
-        const uint32_t a0 = e4m3_pair_to_f16x2(x0 << 8), a1 = e4m3_pair_to_f16x2(x1 << 8);
-        const uint32_t a2 = e4m3_pair_to_f16x2(x0), a3 = e4m3_pair_to_f16x2(x1);
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) mma_f16_16816(acc[mt][nt], a0, a1, a2, a3, pb0[nt], pb1[nt]);
       }
 
       // release the stage to the async proxy, then refill it
@@ -346,7 +418,7 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const F8Pools
       for (int e = 0; e < 2; ++e)
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) l_run[nt][e] += __shfl_xor_sync(0xffffffffu, l_run[nt][e], o);
-    const float unit = F >= -126 ? exp2i(-F) : 0.f;  // acc -> output units (F <= 120)
+    const float unit = exp2i(-F);  // acc -> output units (|F| <= 120)
     constexpr int kLd = kHeadDim + 1;
     float* so = scratch;                 // [8*NT][kLd]
     float* sl = scratch + 8 * NT * kLd;  // [8*NT] base-2 lse
@@ -406,24 +478,13 @@ constexpr int kF8AppendWarps = 8;
 struct F8AppendParams {
   const __nv_bfloat16* k_new;  // [T, Hkv, D]
   const __nv_bfloat16* v_new;
-  uint8_t* k8;                 // [P, Hkv, 16, D]
-  uint8_t* v8;                 // [P, Hkv, D, 16]
-  float* k_scale;              // [P, Hkv, 16]
-  float* v_scale;
+  uint8_t* kv8;                // [P, Hkv] blocks of kF8BlockBytes
   const int32_t* block_table;
   const int32_t* seq_lens;
   const int32_t* qsl;
   int32_t* status;
   int32_t num_seqs, total_q, max_pages, num_pages, num_kv_heads;
 };
-
-// The e4m3 codes of x0 (low byte) and x1 (high byte): nearest, ties to
-// even, saturating at +-448.
-__device__ __forceinline__ uint32_t e4m3x2(float x0, float x1) {
-  uint16_t d;
-  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(d) : "f"(x1), "f"(x0));
-  return d;
-}
 
 // one warp per (token, kv head): lane l quantizes dims 2l and 2l + 1 of K and V
 __global__ void __launch_bounds__(kF8AppendWarps * 32) kv_append_fp8_kernel(const F8AppendParams p) {
@@ -458,7 +519,7 @@ __global__ void __launch_bounds__(kF8AppendWarps * 32) kv_append_fp8_kernel(cons
   dst = __shfl_sync(0xffffffffu, dst, 0);
   if (dst < 0) return;
   const int page = dst / kPage, slot = dst % kPage;
-  const size_t blk = (size_t)page * p.num_kv_heads + h;
+  uint8_t* blk = p.kv8 + ((size_t)page * p.num_kv_heads + h) * kF8BlockBytes;
 #pragma unroll
   for (int which = 0; which < 2; ++which) {
     const __nv_bfloat16* src = (which ? p.v_new : p.k_new) + ((size_t)t * p.num_kv_heads + h) * kHeadDim;
@@ -475,30 +536,27 @@ __global__ void __launch_bounds__(kF8AppendWarps * 32) kv_append_fp8_kernel(cons
       code = e4m3x2(__fmul_rn(x0, inv), __fmul_rn(x1, inv));
     }
     if (which == 0) {
-      reinterpret_cast<uint16_t*>(p.k8 + (blk * kPage + slot) * kHeadDim)[lane] = (uint16_t)code;
-      if (lane == 0) p.k_scale[blk * kPage + slot] = scale;
+      reinterpret_cast<uint16_t*>(blk + slot * kHeadDim)[lane] = (uint16_t)code;
+      if (lane == 0) reinterpret_cast<float*>(blk + kF8KsOff)[slot] = scale;
     } else {
-      uint8_t* col = p.v8 + blk * kF8Block + slot;  // transposed block: [dim][key]
+      uint8_t* col = blk + kF8VOff + slot;  // transposed: [dim][key]
       col[(2 * lane) * kPage] = (uint8_t)(code & 0xFF);
       col[(2 * lane + 1) * kPage] = (uint8_t)(code >> 8);
-      if (lane == 0) p.v_scale[blk * kPage + slot] = scale;
+      if (lane == 0) reinterpret_cast<float*>(blk + kF8VsOff)[slot] = scale;
     }
   }
 }
 
 // ------------------------------------------------------------------ launch
 
-cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* k8, void* v8, float* k_scale,
-                                 float* v_scale, const int32_t* block_table, const int32_t* seq_lens,
-                                 const int32_t* qsl, int32_t* status, int32_t num_seqs, int32_t total_q,
-                                 int32_t max_pages, int32_t num_pages, int32_t num_kv_heads, cudaStream_t stream) {
+cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* kv8, const int32_t* block_table,
+                                 const int32_t* seq_lens, const int32_t* qsl, int32_t* status, int32_t num_seqs,
+                                 int32_t total_q, int32_t max_pages, int32_t num_pages, int32_t num_kv_heads,
+                                 cudaStream_t stream) {
   F8AppendParams p;
   p.k_new = static_cast<const __nv_bfloat16*>(k_new);
   p.v_new = static_cast<const __nv_bfloat16*>(v_new);
-  p.k8 = static_cast<uint8_t*>(k8);
-  p.v8 = static_cast<uint8_t*>(v8);
-  p.k_scale = k_scale;
-  p.v_scale = v_scale;
+  p.kv8 = static_cast<uint8_t*>(kv8);
   p.block_table = block_table;
   p.seq_lens = seq_lens;
   p.qsl = qsl;
@@ -514,17 +572,12 @@ cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* k8,
   return cudaGetLastError();
 }
 
-cudaError_t launch_decode_fp8(const void* k8, const void* v8, const float* k_scale, const float* v_scale,
-                              const AttnParams& p, int grid, bool cascade, cudaStream_t stream) {
-  F8Pools pools;
-  pools.k8 = static_cast<const uint8_t*>(k8);
-  pools.v8 = static_cast<const uint8_t*>(v8);
-  pools.k_scale = k_scale;
-  pools.v_scale = v_scale;
+cudaError_t launch_decode_fp8(const void* kv8, const AttnParams& p, int grid, bool cascade, cudaStream_t stream) {
+  const uint8_t* pool = static_cast<const uint8_t*>(kv8);
   if (cascade)
-    decode_fp8_kernel<4><<<grid, kF8Warps * 32, decode_fp8_smem_bytes(), stream>>>(pools, p);
+    decode_fp8_kernel<4><<<grid, kF8Warps * 32, decode_fp8_smem_bytes(), stream>>>(pool, p);
   else
-    decode_fp8_kernel<1><<<grid, kF8Warps * 32, decode_fp8_smem_bytes(), stream>>>(pools, p);
+    decode_fp8_kernel<1><<<grid, kF8Warps * 32, decode_fp8_smem_bytes(), stream>>>(pool, p);
   return cudaGetLastError();
 }
 

@@ -98,11 +98,11 @@ _lib.mcpu_rope_kv_append.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.
 _lib.mcpu_rope_kv_append.restype = ctypes.c_int
 _lib.mcpu_grow_block_tables.argtypes = [_P, _P, ctypes.POINTER(Dims), _P, _P, _P, _P]
 _lib.mcpu_grow_block_tables.restype = ctypes.c_int
-_lib.mcpu_kv_append_fp8.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.POINTER(Dims), _P, _P]
+_lib.mcpu_kv_append_fp8.argtypes = [_P, _P, _P, _P, _P, _P, ctypes.POINTER(Dims), _P, _P]
 _lib.mcpu_kv_append_fp8.restype = ctypes.c_int
 _lib.mcpu_paged_attention_forward_fp8.argtypes = [
-    _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P,
-    ctypes.c_size_t, ctypes.POINTER(Options), _P,
+    _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P, ctypes.c_size_t,
+    ctypes.POINTER(Options), _P,
 ]
 _lib.mcpu_paged_attention_forward_fp8.restype = ctypes.c_int
 _lib.mcpu_read_device_status.argtypes = [_P, _P, ctypes.POINTER(ctypes.c_int32)]
@@ -262,40 +262,45 @@ def mcpu_paged_attention_forward_noalloc(q, k_cache, v_cache, block_table, seq_l
     )
 
 
-def mcpu_kv_append_fp8(k_new, v_new, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc,
-                       status_word, stream=None):
-    """Quantizing KV append into fp8 pools: k8 uint8 [P, Hkv, 16, D], v8 uint8
-    [P, Hkv, D, 16] (each block transposed), scales float32 [P, Hkv, 16]."""
-    d = Dims(
-        num_seqs=int(seq_lens.shape[0]),
-        total_q=int(k_new.shape[0]),
-        max_pages_per_seq=int(block_table.shape[1]),
-        num_pages=int(k8.shape[0]),
-        num_q_heads=int(k8.shape[1]),
-        num_kv_heads=int(k8.shape[1]),
-        head_dim=int(k8.shape[3]),
-        page_size=int(k8.shape[2]),
-    )
+FP8_BLOCK_BYTES = 2176  # one (page, kv head) block: K codes, V codes (transposed), K and V scales
+
+
+def new_fp8_pool(num_pages, num_kv_heads, device="cuda") -> torch.Tensor:
+    """An (uninitialised) fp8 KV pool: uint8 [num_pages, H_kv, 2176]."""
+    return torch.empty((num_pages, num_kv_heads, FP8_BLOCK_BYTES), dtype=torch.uint8, device=device)
+
+
+def dims_fp8(q, kv8, block_table, seq_lens) -> Dims:
+    """mcpu_dims for an fp8 pool kv8 [P, Hkv, 2176]."""
+    if kv8.dim() != 3 or kv8.shape[2] != FP8_BLOCK_BYTES or kv8.dtype != torch.uint8:
+        raise ValueError("kv8 must be a uint8 [num_pages, H_kv, 2176] tensor")
+    return Dims(num_seqs=int(seq_lens.shape[0]), total_q=int(q.shape[0]), max_pages_per_seq=int(block_table.shape[1]),
+                num_pages=int(kv8.shape[0]), num_q_heads=int(q.shape[1]), num_kv_heads=int(kv8.shape[1]),
+                head_dim=int(q.shape[2]), page_size=16)
+
+
+def mcpu_kv_append_fp8(k_new, v_new, kv8, block_table, seq_lens, query_start_loc, status_word, stream=None):
+    """Quantizing KV append into an fp8 pool kv8 (uint8 [P, Hkv, 2176])."""
+    d = dims_fp8(k_new, kv8, block_table, seq_lens)
+    d.num_q_heads = d.num_kv_heads
     _check(
-        _lib.mcpu_kv_append_fp8(_ptr(k_new), _ptr(v_new), _ptr(k8), _ptr(v8), _ptr(k_scale), _ptr(v_scale),
-                                _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc), ctypes.byref(d),
-                                _ptr(status_word), _stream(stream)),
+        _lib.mcpu_kv_append_fp8(_ptr(k_new), _ptr(v_new), _ptr(kv8), _ptr(block_table), _ptr(seq_lens),
+                                _ptr(query_start_loc), ctypes.byref(d), _ptr(status_word), _stream(stream)),
         "mcpu_kv_append_fp8",
     )
 
 
-def mcpu_paged_attention_forward_fp8(q, k8, v8, k_scale, v_scale, block_table, seq_lens, query_start_loc,
-                                     sliding_window, softmax_scale, out, lse, workspace, flags=0, split_pages=0,
-                                     stream=None, phase_events=None, sinks=None):
-    """Decode-row attention over fp8 pools (layouts as mcpu_kv_append_fp8)."""
-    d = dims(q, k8, block_table, seq_lens)
+def mcpu_paged_attention_forward_fp8(q, kv8, block_table, seq_lens, query_start_loc, sliding_window, softmax_scale,
+                                     out, lse, workspace, flags=0, split_pages=0, stream=None, phase_events=None,
+                                     sinks=None):
+    """Decode-row attention over an fp8 pool (layout as mcpu_kv_append_fp8)."""
+    d = dims_fp8(q, kv8, block_table, seq_lens)
     opts = _options(d.num_q_heads, flags, split_pages, phase_events, sinks)
     _check(
         _lib.mcpu_paged_attention_forward_fp8(
-            _ptr(q), _ptr(k8), _ptr(v8), _ptr(k_scale), _ptr(v_scale), _ptr(block_table), _ptr(seq_lens),
-            _ptr(query_start_loc), int(sliding_window), float(softmax_scale), ctypes.byref(d), _ptr(out), _ptr(lse),
-            _ptr(workspace), int(workspace.numel() * workspace.element_size()), ctypes.byref(opts),
-            _stream(stream),
+            _ptr(q), _ptr(kv8), _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc), int(sliding_window),
+            float(softmax_scale), ctypes.byref(d), _ptr(out), _ptr(lse), _ptr(workspace),
+            int(workspace.numel() * workspace.element_size()), ctypes.byref(opts), _stream(stream),
         ),
         "mcpu_paged_attention_forward_fp8",
     )

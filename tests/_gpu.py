@@ -137,9 +137,28 @@ def oracle_quantize_pool(k_bits, v_bits):
     return oracle.kv_append_fp8(tok(k_bits), tok(v_bits), z8, z8, zs, zs, bt, sl, qsl)
 
 
-def v_to_device_layout(v8):
-    """Oracle V codes [P, Hkv, 16, D] -> the ABI's transposed blocks [P, Hkv, D, 16]."""
-    return np.ascontiguousarray(np.asarray(v8).transpose(0, 1, 3, 2))
+def to_fp8_blocks(k8, v8, ks, vs):
+    """Oracle arrays (codes [P, Hkv, 16, D], scales [P, Hkv, 16]) -> the
+    ABI's pool of 2176-byte blocks [P, Hkv, 2176]: K codes, V codes
+    transposed to [D][16], K scales, V scales."""
+    P, H, page, D = k8.shape
+    blk = np.empty((P, H, 2176), np.uint8)
+    blk[..., :1024] = np.asarray(k8).reshape(P, H, page * D)
+    blk[..., 1024:2048] = np.asarray(v8).transpose(0, 1, 3, 2).reshape(P, H, page * D)
+    blk[..., 2048:2112] = np.ascontiguousarray(ks, dtype=np.float32).view(np.uint8).reshape(P, H, 64)
+    blk[..., 2112:2176] = np.ascontiguousarray(vs, dtype=np.float32).view(np.uint8).reshape(P, H, 64)
+    return blk
+
+
+def from_fp8_blocks(blk):
+    """Inverse of to_fp8_blocks."""
+    blk = np.asarray(blk)
+    P, H, _ = blk.shape
+    k8 = blk[..., :1024].reshape(P, H, 16, 64)
+    v8 = blk[..., 1024:2048].reshape(P, H, 64, 16).transpose(0, 1, 3, 2)
+    ks = np.ascontiguousarray(blk[..., 2048:2112]).view(np.float32).reshape(P, H, 16)
+    vs = np.ascontiguousarray(blk[..., 2112:2176]).view(np.float32).reshape(P, H, 16)
+    return np.ascontiguousarray(k8), np.ascontiguousarray(v8), ks, vs
 
 
 class Fp8Run:
@@ -172,23 +191,20 @@ class Fp8Run:
         self.q = lay.q.to(dev)
         self.k_new = lay.k_new.to(dev)
         self.v_new = lay.v_new.to(dev)
-        self.k8 = torch.from_numpy(k8).to(dev)
-        self.v8 = torch.from_numpy(v_to_device_layout(v8)).to(dev)
-        self.ks = torch.from_numpy(ks).to(dev)
-        self.vs = torch.from_numpy(vs).to(dev)
+        self.kv8 = torch.from_numpy(to_fp8_blocks(k8, v8, ks, vs)).to(dev)
         pool = batch.pools[lay.pool]
         self.bt = torch.from_numpy(pool.block_table).to(dev)
         self.sl = torch.from_numpy(batch.seq_lens).to(dev)
         self.qsl = torch.from_numpy(batch.query_start_loc).to(dev)
         self.window = lay.sliding_window
-        self.dims = mcpu.dims(self.q, self.k8, self.bt, self.sl)
+        self.dims = mcpu.dims_fp8(self.q, self.kv8, self.bt, self.sl)
         self.ws = mcpu.new_workspace(self.dims, dev)
         self.out = torch.full_like(self.q, float("nan"))
         self.lse = torch.full(self.q.shape[:2], float("nan"), dtype=torch.float32, device=dev)
 
     def append(self):
-        mcpu.mcpu_kv_append_fp8(self.k_new, self.v_new, self.k8, self.v8, self.ks, self.vs, self.bt, self.sl,
-                                self.qsl, mcpu.status_word(self.ws))
+        mcpu.mcpu_kv_append_fp8(self.k_new, self.v_new, self.kv8, self.bt, self.sl, self.qsl,
+                                mcpu.status_word(self.ws))
 
     def oracle_append(self):
         h = self.h
@@ -197,9 +213,9 @@ class Fp8Run:
 
     def forward(self, flags=0, split_pages=0, sinks=None):
         sk = None if sinks is None else torch.from_numpy(np.asarray(sinks, np.float32)).to(self.q.device)
-        mcpu.mcpu_paged_attention_forward_fp8(self.q, self.k8, self.v8, self.ks, self.vs, self.bt, self.sl,
-                                              self.qsl, self.window, self.batch.softmax_scale, self.out, self.lse,
-                                              self.ws, flags=flags, split_pages=split_pages, sinks=sk)
+        mcpu.mcpu_paged_attention_forward_fp8(self.q, self.kv8, self.bt, self.sl, self.qsl, self.window,
+                                              self.batch.softmax_scale, self.out, self.lse, self.ws, flags=flags,
+                                              split_pages=split_pages, sinks=sk)
 
     def status(self):
         return mcpu.mcpu_read_device_status(self.ws)
@@ -210,7 +226,8 @@ class Fp8Run:
                     n_merge=int(hd[4]), split_pages=int(hd[5]), n_parts=int(hd[6]))
 
     def pools_host(self):
-        return (self.k8.cpu().numpy(), self.v8.cpu().numpy(), self.ks.cpu().numpy(), self.vs.cpu().numpy())
+        """The device pool as oracle arrays (k8, v8, k_scale, v_scale)."""
+        return from_fp8_blocks(self.kv8.cpu().numpy())
 
     def out_host(self):
         return self.out.float().cpu().numpy(), self.lse.cpu().numpy()

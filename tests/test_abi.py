@@ -119,27 +119,28 @@ def test_kv_append_host_validation(lib):
 
 def test_fp8_host_validation(lib):
     fwd = _fn(lib, "mcpu_paged_attention_forward_fp8")
-    fwd.argtypes = [ctypes.c_void_p] * 8 + [ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims)] + \
+    fwd.argtypes = [ctypes.c_void_p] * 5 + [ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims)] + \
         [ctypes.c_void_p] * 3 + [ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]
     d = Dims(4, 4, 19, 34, 8, 2, 64, 16)
     P = 1 << 20
     lib.mcpu_workspace_size.restype = ctypes.c_size_t
     need = lib.mcpu_workspace_size(ctypes.byref(d))
-    args = [P] * 8 + [0, 0.125, ctypes.byref(d), P, P, P, need, None, None]
-    a = list(args); a[3] = None           # no k_scale
+    args = [P] * 5 + [0, 0.125, ctypes.byref(d), P, P, P, need, None, None]
+    a = list(args); a[1] = None           # no pool
     assert fwd(*a) == 1
-    a = list(args); a[4] = P + 4          # misaligned v_scale
+    a = list(args); a[1] = P + 8          # misaligned pool
     assert fwd(*a) == 1
     d_app = Dims(4, 9, 19, 34, 8, 2, 64, 16)  # 9 query tokens over 4 rows: some row appends
-    a = list(args); a[10] = ctypes.byref(d_app); a[14] = lib.mcpu_workspace_size(ctypes.byref(d_app))
+    a = list(args); a[7] = ctypes.byref(d_app); a[11] = lib.mcpu_workspace_size(ctypes.byref(d_app))
     assert fwd(*a) == 2
     d0 = Dims(0, 0, 19, 34, 8, 2, 64, 16)
-    a = list(args); a[10] = ctypes.byref(d0); a[14] = lib.mcpu_workspace_size(ctypes.byref(d0))
+    a = list(args); a[7] = ctypes.byref(d0); a[11] = lib.mcpu_workspace_size(ctypes.byref(d0))
     assert fwd(*a) == 0
     app = _fn(lib, "mcpu_kv_append_fp8")
-    app.argtypes = [ctypes.c_void_p] * 9 + [ctypes.POINTER(Dims), ctypes.c_void_p, ctypes.c_void_p]
-    assert app(P, P, P, P, P, None, P, P, P, ctypes.byref(d), P, None) == 1   # no v_scale
-    assert app(P, P, P, P + 8, P, P, P, P, P, ctypes.byref(d), P, None) == 1  # misaligned v8
+    app.argtypes = [ctypes.c_void_p] * 6 + [ctypes.POINTER(Dims), ctypes.c_void_p, ctypes.c_void_p]
+    assert app(P, P, None, P, P, P, ctypes.byref(d), P, None) == 1   # no pool
+    assert app(P, P, P + 4, P, P, P, ctypes.byref(d), P, None) == 1  # misaligned pool
+    assert app(P, P, P, P, P, P, ctypes.byref(d), None, None) == 1   # no status word
 
 
 def test_status_strings(lib):
