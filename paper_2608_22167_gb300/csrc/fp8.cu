@@ -3,10 +3,15 @@
 //
 // Storage: one 2176-byte block per (page, kv head), blocks ordered
 // [page][kv head]:
-//   bytes    0..1023  K codes [16 keys][64 dims]  (row-major)
-//   bytes 1024..2047  V codes [64 dims][16 keys]  (transposed)
-//   bytes 2048..2111  K scales [16] float
-//   bytes 2112..2175  V scales [16] float
+//   bytes    0..1023  K codes [16 keys][64 dims] (row-major)
+//   bytes 1024..2047  V codes in MMA-fragment order: for h in {0, 1}, lane
+//                     (r, c) = (l / 4, l % 4) and j in 0..3, bytes
+//                     1024 + 512 h + 16 l + 4 j + i hold dim
+//                     d = 16 (2h + j / 2) + 8 (j % 2) + r of key 4c + i
+//   bytes 2048..2175  scales: 16 bytes per r in 0..7 = K scale of keys
+//                     a = 4(r / 2) + r % 2 and a + 2, then V scale of both
+// so that one bulk copy brings a page and every operand of a lane is one
+// 128-bit shared-memory load (two for K, two for V, one for the scales).
 // Each new row x (64 bf16 values) is stored as a = max|x_i|, scale = a / 448
 // and code_i = e4m3(x_i * (448 / a)) (round to nearest even, saturating), in
 // float arithmetic; an all-zero row stores zeros. A key is code * scale.
@@ -23,15 +28,21 @@
 //     page). Each score is then scaled by its key's scale, the power of two
 //     and the softmax scale;
 //   - O += P' V: P' = p * v_scale * 2^F in fp16 (F a per-item power of two
-//     that only decreases, so that P' < 2^8) is split into e4m3 hi + lo, the
+//     that only decreases, so that v_scale * 2^F < 1 and P' < 2^8) is
+//     split into e4m3 hi + lo, the
 //     two pieces sit in the two halves of the MMA's k range beside a
 //     duplicated V operand (4 MMAs per page). The accumulator is rescaled
 //     when F drops and divided by 2^F at the end.
 // Which keys meet in which MMA row/slot is a permutation chosen so that the
 // score fragment transposes into the P' operand with movmatrix: M row r of
-// the score tile is key 4(r/2) + (r%2), row r + 8 is that key + 2. V codes of
-// keys a row cannot see are zeroed in registers (unwritten slots may hold
-// any byte, e4m3 NaN included); a page outside the pool is skipped.
+// the score tile is key 4(r/2) + (r%2), row r + 8 is that key + 2. The
+// running max is lazy: scores are exponentiated against a reference that
+// is only raised (with the rescale) when a score exceeds it by more than 8
+// (p <= 2^8), and F is only lowered when a page's V scale needs it; both
+// checks are one warp vote per page. On pages that a row sees only in part
+// (its first and last), V codes of invisible keys are zeroed in registers
+// (unwritten slots may hold any byte, e4m3 NaN included); a page outside
+// the pool is skipped.
 #include <cuda_fp16.h>
 
 #include "common.cuh"
@@ -39,12 +50,13 @@
 namespace mcpu {
 
 constexpr int kF8Warps = 4;
-constexpr int kF8Stages = 8;
+constexpr int kF8Stages = 6;
 constexpr int kF8Codes = kPage * kHeadDim;  // 1024 codes per (page, kv head) for K, and for V
 constexpr int kF8VOff = kF8Codes;
-constexpr int kF8KsOff = 2 * kF8Codes;
-constexpr int kF8VsOff = 2 * kF8Codes + kPage * 4;
+constexpr int kF8ScaleOff = 2 * kF8Codes;
 constexpr int kF8BlockBytes = 2 * kF8Codes + 2 * kPage * 4;  // 2176
+constexpr float kF8Lazy = 8.f;      // scores may exceed the reference max by this much (base 2)
+constexpr float kF8NoMax = -1e30f;  // reference max before the first visible key
 constexpr int kF8RingBytes = kF8Stages * kF8BlockBytes;
 
 size_t decode_fp8_smem_bytes() {
@@ -114,7 +126,7 @@ __device__ __forceinline__ uint32_t key_byte_mask(int c, int lo, int hi) {
 }
 
 template <int NT>
-__global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t* __restrict__ kv8,
+__global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_kernel(const uint8_t* __restrict__ kv8,
                                                                    const AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -258,9 +270,8 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
       }
       return __shfl_sync(0xffffffffu, pid_reg, k & 31);
     };
-    auto issue = [&](int k) {
+    auto issue = [&](int k, uint32_t s) {  // page k of the item into ring stage s
       const int pid = page_id(k);
-      const uint32_t s = (seq + k) % kF8Stages;
       bad_stages = pid < 0 ? (bad_stages | (1u << s)) : (bad_stages & ~(1u << s));
       if (lane == 0) {
         const uint32_t bar = bars + 8 * s;
@@ -274,24 +285,25 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
       }
     };
     const int pre = n < kF8Stages ? n : kF8Stages;
-    for (int k = 0; k < pre; ++k) issue(k);
+    for (int k = 0; k < pre; ++k) issue(k, (seq + k) % kF8Stages);
 
-    float m_run[NT][2], l_run[NT][2], acc[4][NT][4];
+    float m_ref[NT][2], l_run[NT][2], acc[4][NT][4];
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
-      m_run[nt][0] = m_run[nt][1] = -INFINITY;
+      m_ref[nt][0] = m_ref[nt][1] = kF8NoMax;
       l_run[nt][0] = l_run[nt][1] = 0.f;
 #pragma unroll
       for (int mt = 0; mt < 4; ++mt)
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
     }
-    int F = 120;  // P' = p * v_scale * 2^F; acc is held in units of 2^F
+    int F = 125;           // P' = p * v_scale * 2^F; acc is held in units of 2^F
+    float u_lim = 0.f;     // 2^-F: a V scale at or above it needs a lower F
+    float pf = exp2i(F);
 
     bool timed_out = false;
+    uint32_t s = seq % kF8Stages, phase = (seq / kF8Stages) & 1u;
     for (int k = 0; k < n; ++k) {
-      const uint32_t s = (seq + k) % kF8Stages;
-      const uint32_t phase = ((seq + k) / kF8Stages) & 1u;
       const bool ok = __any_sync(0xffffffffu, mbar_wait(bars + 8 * s, phase));
       if (!ok) {
         timed_out = true;
@@ -301,9 +313,9 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
         const uint8_t* st = ring_ptr + s * kF8BlockBytes;
         const uint4 KA = *reinterpret_cast<const uint4*>(st + key_a * kHeadDim + 16 * c);
         const uint4 KB = *reinterpret_cast<const uint4*>(st + key_b * kHeadDim + 16 * c);
-        const float* ksp = reinterpret_cast<const float*>(st + kF8KsOff);
-        const float* vsp = reinterpret_cast<const float*>(st + kF8VsOff);
-        const float ks0 = ksp[key_a], ks1 = ksp[key_b], vs0 = vsp[key_a], vs1 = vsp[key_b];
+        const float4 sc = *reinterpret_cast<const float4*>(st + kF8ScaleOff + 16 * r);  // ks_a, ks_b, vs_a, vs_b
+        const uint4 V0 = *reinterpret_cast<const uint4*>(st + kF8VOff + 16 * lane);
+        const uint4 V1 = *reinterpret_cast<const uint4*>(st + kF8VOff + 512 + 16 * lane);
 
         // S^T[16 keys x 8*NT query vectors] in units of q * 2^eq * K codes
         float cc[NT][4];
@@ -322,58 +334,84 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
           }
         }
 
-        // visible keys of this page: [klo, khi)
-        const int pk = (pb + k) * kPage;
-        int klo = 0, khi = kPage;
-        if (NT == 1) {
-          klo = max(first_key - pk, 0);
-          khi = min(seq_len - pk, kPage);
+        float sv[NT][4];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          sv[nt][0] = cc[nt][0] * (sc.x * qm[nt][0]);
+          sv[nt][1] = cc[nt][1] * (sc.x * qm[nt][1]);
+          sv[nt][2] = cc[nt][2] * (sc.y * qm[nt][0]);
+          sv[nt][3] = cc[nt][3] * (sc.y * qm[nt][1]);
         }
-        const bool v0 = key_a >= klo && key_a < khi, v1 = key_b >= klo && key_b < khi;
-        // the page's power of two for P' (F only decreases)
-        const float u0 = v0 ? vs0 : 0.f, u1 = v1 ? vs1 : 0.f;
-        float umax = fmaxf(u0, u1);
-        umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 4));
-        umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 8));
-        umax = fmaxf(umax, __shfl_xor_sync(0xffffffffu, umax, 16));
-        int F_new = F;
-        if (umax > 0.f) F_new = min(F, max(7 - ilog2f(umax), -120));
-        const float dF = F_new < F ? (F_new - F >= -126 ? exp2i(F_new - F) : 0.f) : 1.f;
-        F = F_new;
-        const float pf = exp2i(F);
+        float u0 = sc.z, u1 = sc.w;
+        uint32_t vmask = 0xFFFFFFFFu;
+        // a row's first and last pages may hold keys it does not see
+        const int pk = (pb + k) * kPage;
+        if (NT == 1 && (pk < first_key || pk + kPage > seq_len)) {
+          const int klo = max(first_key - pk, 0), khi = min(seq_len - pk, kPage);
+          const bool v0 = key_a >= klo && key_a < khi, v1 = key_b >= klo && key_b < khi;
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            sv[nt][0] = v0 ? sv[nt][0] : -INFINITY;
+            sv[nt][1] = v0 ? sv[nt][1] : -INFINITY;
+            sv[nt][2] = v1 ? sv[nt][2] : -INFINITY;
+            sv[nt][3] = v1 ? sv[nt][3] : -INFINITY;
+          }
+          u0 = v0 ? u0 : 0.f;
+          u1 = v1 ? u1 : 0.f;
+          vmask = key_byte_mask(c, klo, khi);
+        }
+
+        // rare: a score above the reference by more than kF8Lazy, or a V
+        // scale that needs a lower F
+        bool over = fmaxf(u0, u1) >= u_lim;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+          over |= fmaxf(sv[nt][0], sv[nt][2]) > m_ref[nt][0] + kF8Lazy ||
+                  fmaxf(sv[nt][1], sv[nt][3]) > m_ref[nt][1] + kF8Lazy;
+        if (__any_sync(0xffffffffu, over)) {
+          float um = fmaxf(u0, u1);
+          um = fmaxf(um, __shfl_xor_sync(0xffffffffu, um, 4));
+          um = fmaxf(um, __shfl_xor_sync(0xffffffffu, um, 8));
+          um = fmaxf(um, __shfl_xor_sync(0xffffffffu, um, 16));
+          int F_new = F;
+          if (um >= u_lim && um > 0.f) F_new = max(min(F, -1 - ilog2f(um)), -125);
+          const float dF = F_new - F >= -126 ? exp2i(F_new - F) : 0.f;
+          F = F_new;
+          pf = exp2i(F);
+          u_lim = exp2i(-F);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            float mx0 = fmaxf(sv[nt][0], sv[nt][2]), mx1 = fmaxf(sv[nt][1], sv[nt][3]);
+#pragma unroll
+            for (int o = 4; o < 32; o <<= 1) {
+              mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+              mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+            }
+            const float mn0 = fmaxf(m_ref[nt][0], mx0), mn1 = fmaxf(m_ref[nt][1], mx1);
+            const float al0 = ex2_approx(m_ref[nt][0] - mn0), al1 = ex2_approx(m_ref[nt][1] - mn1);
+            m_ref[nt][0] = mn0;
+            m_ref[nt][1] = mn1;
+            l_run[nt][0] *= al0;
+            l_run[nt][1] *= al1;
+            const float ac0 = al0 * dF, ac1 = al1 * dF;
+#pragma unroll
+            for (int mt = 0; mt < 4; ++mt) {
+              acc[mt][nt][0] *= ac0;
+              acc[mt][nt][1] *= ac1;
+              acc[mt][nt][2] *= ac0;
+              acc[mt][nt][3] *= ac1;
+            }
+          }
+        }
         const float w0 = u0 * pf, w1 = u1 * pf;
 
         uint32_t pv_hi[NT], pv_lo[NT];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
-          const float s00 = v0 ? cc[nt][0] * ks0 * qm[nt][0] : -INFINITY;
-          const float s01 = v0 ? cc[nt][1] * ks0 * qm[nt][1] : -INFINITY;
-          const float s10 = v1 ? cc[nt][2] * ks1 * qm[nt][0] : -INFINITY;
-          const float s11 = v1 ? cc[nt][3] * ks1 * qm[nt][1] : -INFINITY;
-          float mx0 = fmaxf(s00, s10), mx1 = fmaxf(s01, s11);
-#pragma unroll
-          for (int o = 4; o < 32; o <<= 1) {
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-          }
-          const float mn0 = fmaxf(m_run[nt][0], mx0), mn1 = fmaxf(m_run[nt][1], mx1);
-          const float mu0 = mn0 == -INFINITY ? 0.f : mn0;
-          const float mu1 = mn1 == -INFINITY ? 0.f : mn1;
-          const float al0 = fast_exp2(m_run[nt][0] - mu0), al1 = fast_exp2(m_run[nt][1] - mu1);
-          const float p00 = fast_exp2(s00 - mu0), p10 = fast_exp2(s10 - mu0);
-          const float p01 = fast_exp2(s01 - mu1), p11 = fast_exp2(s11 - mu1);
-          l_run[nt][0] = l_run[nt][0] * al0 + p00 + p10;
-          l_run[nt][1] = l_run[nt][1] * al1 + p01 + p11;
-          m_run[nt][0] = mn0;
-          m_run[nt][1] = mn1;
-          const float ac0 = al0 * dF, ac1 = al1 * dF;
-#pragma unroll
-          for (int mt = 0; mt < 4; ++mt) {
-            acc[mt][nt][0] *= ac0;
-            acc[mt][nt][1] *= ac1;
-            acc[mt][nt][2] *= ac0;
-            acc[mt][nt][3] *= ac1;
-          }
+          const float p00 = ex2_approx(sv[nt][0] - m_ref[nt][0]), p01 = ex2_approx(sv[nt][1] - m_ref[nt][1]);
+          const float p10 = ex2_approx(sv[nt][2] - m_ref[nt][0]), p11 = ex2_approx(sv[nt][3] - m_ref[nt][1]);
+          l_run[nt][0] += p00 + p10;
+          l_run[nt][1] += p01 + p11;
           // P' in fp16, split into e4m3 hi + lo; each key's (hi, lo) codes
           // form one 16-bit element for the transpose
           const uint32_t fa = pack_f16x2(p00 * w0, p01 * w0), fb = pack_f16x2(p10 * w1, p11 * w1);
@@ -387,24 +425,28 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
         }
 
         // O^T[64 dims x 8*NT] += V^T P'^T: k-slots 0..15 carry the hi piece,
-        // 16..31 the lo piece, both against the same V codes
-        const uint32_t vmask = (klo > 0 || khi < kPage) ? key_byte_mask(c, klo, khi) : 0xFFFFFFFFu;
+        // 16..31 the lo piece, both against the same V codes (dims
+        // 16 mt + r and 16 mt + 8 + r, keys 4c .. 4c + 3)
+        const uint32_t vw[8] = {V0.x & vmask, V0.y & vmask, V0.z & vmask, V0.w & vmask,
+                                V1.x & vmask, V1.y & vmask, V1.z & vmask, V1.w & vmask};
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
-          const uint32_t x0 = *reinterpret_cast<const uint32_t*>(st + kF8VOff + (16 * mt + r) * kPage + 4 * c) & vmask;
-          const uint32_t x1 =
-              *reinterpret_cast<const uint32_t*>(st + kF8VOff + (16 * mt + r + 8) * kPage + 4 * c) & vmask;
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) mma_e4m3_16832(acc[mt][nt], x0, x1, x0, x1, pv_hi[nt], pv_lo[nt]);
+          for (int nt = 0; nt < NT; ++nt)
+            mma_e4m3_16832(acc[mt][nt], vw[2 * mt], vw[2 * mt + 1], vw[2 * mt], vw[2 * mt + 1], pv_hi[nt],
+                           pv_lo[nt]);
         }
       }
 
       // release the stage to the async proxy, then refill it
       fence_proxy_async();
       __syncwarp();
-      if (k + kF8Stages < n) issue(k + kF8Stages);
+      if (k + kF8Stages < n) issue(k + kF8Stages, s);
+      if (++s == kF8Stages) {
+        s = 0;
+        phase ^= 1u;
+      }
     }
-
     if (timed_out) {
       raise_status(p, kStatusTimeout);
       return;  // the ring's phase tracking is lost: this warp stops here
@@ -418,7 +460,7 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
       for (int e = 0; e < 2; ++e)
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) l_run[nt][e] += __shfl_xor_sync(0xffffffffu, l_run[nt][e], o);
-    const float unit = exp2i(-F);  // acc -> output units (|F| <= 120)
+    const float unit = exp2i(-F);  // acc -> output units (|F| <= 125)
     constexpr int kLd = kHeadDim + 1;
     float* so = scratch;                 // [8*NT][kLd]
     float* sl = scratch + 8 * NT * kLd;  // [8*NT] base-2 lse
@@ -428,10 +470,11 @@ __global__ void __launch_bounds__(kF8Warps * 32) decode_fp8_kernel(const uint8_t
       for (int e = 0; e < 2; ++e) {
         const int qv = nt * 8 + 2 * c + e;
         const float l = l_run[nt][e];
+        const float m = l > 0.f ? m_ref[nt][e] : -INFINITY;
         float inv = l > 0.f ? 1.f / l : 0.f;
-        float lse2 = l > 0.f ? m_run[nt][e] + __log2f(l) : -INFINITY;
+        float lse2 = l > 0.f ? m + __log2f(l) : -INFINITY;
         if (NT == 1 && p.sinks != nullptr && slot < 0 && qv < g)
-          inv = finish_with_sink(m_run[nt][e], l, sink_log2(p, kvh * g + qv), &lse2);
+          inv = finish_with_sink(m, l, sink_log2(p, kvh * g + qv), &lse2);
         inv *= unit;
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
@@ -535,14 +578,19 @@ __global__ void __launch_bounds__(kF8AppendWarps * 32) kv_append_fp8_kernel(cons
       scale = __fdiv_rn(a, 448.f);
       code = e4m3x2(__fmul_rn(x0, inv), __fmul_rn(x1, inv));
     }
+    // scale slot of this key: r = 2 (slot / 4) + slot % 2, the key's half (slot / 2) % 2
+    const int sc_idx = 4 * (2 * (slot >> 2) + (slot & 1)) + ((slot >> 1) & 1);
     if (which == 0) {
       reinterpret_cast<uint16_t*>(blk + slot * kHeadDim)[lane] = (uint16_t)code;
-      if (lane == 0) reinterpret_cast<float*>(blk + kF8KsOff)[slot] = scale;
+      if (lane == 0) reinterpret_cast<float*>(blk + kF8ScaleOff)[sc_idx] = scale;
     } else {
-      uint8_t* col = blk + kF8VOff + slot;  // transposed: [dim][key]
-      col[(2 * lane) * kPage] = (uint8_t)(code & 0xFF);
-      col[(2 * lane + 1) * kPage] = (uint8_t)(code >> 8);
-      if (lane == 0) reinterpret_cast<float*>(blk + kF8VsOff)[slot] = scale;
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {  // dim d = 2 lane + e in fragment order
+        const int d = 2 * lane + e, mt = d >> 4, hf = (d >> 3) & 1, rr = d & 7;
+        const int off = kF8VOff + (mt >> 1) * 512 + (4 * rr + (slot >> 2)) * 16 + 4 * ((mt & 1) * 2 + hf) + (slot & 3);
+        blk[off] = (uint8_t)(e ? code >> 8 : code & 0xFF);
+      }
+      if (lane == 0) reinterpret_cast<float*>(blk + kF8ScaleOff)[sc_idx + 2] = scale;
     }
   }
 }

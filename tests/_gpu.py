@@ -137,16 +137,41 @@ def oracle_quantize_pool(k_bits, v_bits):
     return oracle.kv_append_fp8(tok(k_bits), tok(v_bits), z8, z8, zs, zs, bt, sl, qsl)
 
 
+def _fp8_v_order():
+    """Byte position, inside the V area of a block, of (dim d, key j): the
+    MMA-fragment order of the ABI (half h, lane 4r + c, word j', byte i)."""
+    pos = np.empty((64, 16), np.int64)
+    for d in range(64):
+        mt, hf, r = d >> 4, (d >> 3) & 1, d & 7
+        for key in range(16):
+            c, i = key >> 2, key & 3
+            pos[d, key] = (mt >> 1) * 512 + (4 * r + c) * 16 + 4 * ((mt & 1) * 2 + hf) + i
+    return pos
+
+
+def _fp8_scale_order():
+    """Float index, inside the scale area, of the K scale of key j (the V
+    scale sits two floats later): 16 bytes per r = 2 (j / 4) + j % 2."""
+    j = np.arange(16)
+    return 4 * (2 * (j >> 2) + (j & 1)) + ((j >> 1) & 1)
+
+
 def to_fp8_blocks(k8, v8, ks, vs):
     """Oracle arrays (codes [P, Hkv, 16, D], scales [P, Hkv, 16]) -> the
-    ABI's pool of 2176-byte blocks [P, Hkv, 2176]: K codes, V codes
-    transposed to [D][16], K scales, V scales."""
+    ABI's pool of 2176-byte blocks [P, Hkv, 2176]."""
     P, H, page, D = k8.shape
-    blk = np.empty((P, H, 2176), np.uint8)
+    blk = np.zeros((P, H, 2176), np.uint8)
     blk[..., :1024] = np.asarray(k8).reshape(P, H, page * D)
-    blk[..., 1024:2048] = np.asarray(v8).transpose(0, 1, 3, 2).reshape(P, H, page * D)
-    blk[..., 2048:2112] = np.ascontiguousarray(ks, dtype=np.float32).view(np.uint8).reshape(P, H, 64)
-    blk[..., 2112:2176] = np.ascontiguousarray(vs, dtype=np.float32).view(np.uint8).reshape(P, H, 64)
+    vpos = _fp8_v_order()  # [D, 16]
+    vt = np.asarray(v8).transpose(0, 1, 3, 2)  # [P, H, D, 16]
+    varea = np.zeros((P, H, 1024), np.uint8)
+    varea[..., vpos.reshape(-1)] = vt.reshape(P, H, -1)
+    blk[..., 1024:2048] = varea
+    sidx = _fp8_scale_order()
+    sc = np.zeros((P, H, 32), np.float32)
+    sc[..., sidx] = ks
+    sc[..., sidx + 2] = vs
+    blk[..., 2048:2176] = sc.view(np.uint8).reshape(P, H, 128)
     return blk
 
 
@@ -155,10 +180,11 @@ def from_fp8_blocks(blk):
     blk = np.asarray(blk)
     P, H, _ = blk.shape
     k8 = blk[..., :1024].reshape(P, H, 16, 64)
-    v8 = blk[..., 1024:2048].reshape(P, H, 64, 16).transpose(0, 1, 3, 2)
-    ks = np.ascontiguousarray(blk[..., 2048:2112]).view(np.float32).reshape(P, H, 16)
-    vs = np.ascontiguousarray(blk[..., 2112:2176]).view(np.float32).reshape(P, H, 16)
-    return np.ascontiguousarray(k8), np.ascontiguousarray(v8), ks, vs
+    vpos = _fp8_v_order()
+    v8 = blk[..., 1024:2048][..., vpos.reshape(-1)].reshape(P, H, 64, 16).transpose(0, 1, 3, 2)
+    sc = np.ascontiguousarray(blk[..., 2048:2176]).view(np.float32).reshape(P, H, 32)
+    sidx = _fp8_scale_order()
+    return np.ascontiguousarray(k8), np.ascontiguousarray(v8), sc[..., sidx].copy(), sc[..., sidx + 2].copy()
 
 
 class Fp8Run:
