@@ -22,11 +22,14 @@
 // cores (mma m16n8k32, e4m3 x e4m3 -> f32), so the codes go from shared
 // memory into the MMAs as they are:
 //   - S = K q: q (bf16) times a power of two per query vector (largest
-//     entry in [2^7, 2^8)) is split into three e4m3 pieces hi + mid + lo,
-//     exact to ~2^-12 of the largest entry; the hi and mid pieces share one
-//     MMA through a duplicated K operand, lo pieces take two more (6 per
-//     page). Each score is then scaled by its key's scale, the power of two
-//     and the softmax scale;
+//     entry in [2^7, 2^8)) is split into two e4m3 pieces hi + mid. A bf16
+//     value has 8 significant bits, so hi (4 bits, nearest) leaves a
+//     residual that is an integer multiple of 2^-7 of the value's binade
+//     and at most 8 such units: mid holds it exactly unless it falls below
+//     the e4m3 subnormal quantum 2^-9 (entries under 2^-9 of the largest;
+//     their error is at most 2^-17 of it). The two pieces share one MMA
+//     through a duplicated K operand (4 MMAs per page). Each score is then
+//     scaled by its key's scale, the power of two and the softmax scale;
 //   - O += P' V: P' = p * v_scale * 2^F in fp16 (F a per-item power of two
 //     that only decreases, so that v_scale * 2^F < 1 and P' < 2^8) is
 //     split into e4m3 hi + lo, the
@@ -187,10 +190,9 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
     const int* bt_row = p.block_table + (size_t)row * p.max_pages;
 
     // Query vector r (+ 8 nt) as B operands: this lane holds its dims
-    // 16c .. 16c + 15 as e4m3 pieces of q * 2^eq. Step s of the hi/mid MMAs
-    // takes dims 16c + 4s .. + 3 (hi in k-slots 0..15, mid in 16..31); the
-    // two lo MMAs take dims 16c + 8t .. + 3 and 16c + 8t + 4 .. + 3.
-    uint32_t q_hi[NT][4], q_mid[NT][4], q_lo[NT][4];
+    // 16c .. 16c + 15 as e4m3 pieces of q * 2^eq. MMA step j takes dims
+    // 16c + 4j .. + 3, hi in k-slots 0..15 and mid in 16..31.
+    uint32_t q_hi[NT][4], q_mid[NT][4];
     float qm[NT][2];  // score factor of query vectors 2c and 2c + 1
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
@@ -226,23 +228,17 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
       const float up = exp2i(eq);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {  // word j: dims 16c + 4j .. + 3
-        uint32_t h = 0, m = 0, l = 0;
+        uint32_t h = 0, m = 0;
 #pragma unroll
         for (int i = 0; i < 4; i += 2) {
           const float a0 = x[4 * j + i] * up, a1 = x[4 * j + i + 1] * up;
           const uint32_t ch = e4m3x2(a0, a1);
           const float2 vh = e4m3x2_value(ch);
-          const float r0 = a0 - vh.x, r1 = a1 - vh.y;  // exact
-          const uint32_t cm = e4m3x2(r0, r1);
-          const float2 vm = e4m3x2_value(cm);
-          const uint32_t cl = e4m3x2(r0 - vm.x, r1 - vm.y);
           h |= ch << (8 * i);
-          m |= cm << (8 * i);
-          l |= cl << (8 * i);
+          m |= e4m3x2(a0 - vh.x, a1 - vh.y) << (8 * i);  // the residuals are exact in float
         }
         q_hi[nt][j] = h;
         q_mid[nt][j] = m;
-        q_lo[nt][j] = l;
       }
       const float my_qm = exp2i(-eq) * p.scale_log2;
       qm[nt][0] = __shfl_sync(0xffffffffu, my_qm, (2 * c) * 4);
@@ -327,10 +323,6 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
           for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) mma_e4m3_16832(cc[nt], wa[j], wb[j], wa[j], wb[j], q_hi[nt][j], q_mid[nt][j]);
-#pragma unroll
-            for (int t = 0; t < 2; ++t)
-              mma_e4m3_16832(cc[nt], wa[2 * t], wb[2 * t], wa[2 * t + 1], wb[2 * t + 1], q_lo[nt][2 * t],
-                             q_lo[nt][2 * t + 1]);
           }
         }
 
@@ -343,7 +335,7 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
           sv[nt][3] = cc[nt][3] * (sc.y * qm[nt][1]);
         }
         float u0 = sc.z, u1 = sc.w;
-        uint32_t vmask = 0xFFFFFFFFu;
+        uint32_t vw[8] = {V0.x, V0.y, V0.z, V0.w, V1.x, V1.y, V1.z, V1.w};
         // a row's first and last pages may hold keys it does not see
         const int pk = (pb + k) * kPage;
         if (NT == 1 && (pk < first_key || pk + kPage > seq_len)) {
@@ -358,7 +350,9 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
           }
           u0 = v0 ? u0 : 0.f;
           u1 = v1 ? u1 : 0.f;
-          vmask = key_byte_mask(c, klo, khi);
+          const uint32_t vmask = key_byte_mask(c, klo, khi);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) vw[i] &= vmask;
         }
 
         // rare: a score above the reference by more than kF8Lazy, or a V
@@ -427,8 +421,6 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
         // O^T[64 dims x 8*NT] += V^T P'^T: k-slots 0..15 carry the hi piece,
         // 16..31 the lo piece, both against the same V codes (dims
         // 16 mt + r and 16 mt + 8 + r, keys 4c .. 4c + 3)
-        const uint32_t vw[8] = {V0.x & vmask, V0.y & vmask, V0.z & vmask, V0.w & vmask,
-                                V1.x & vmask, V1.y & vmask, V1.z & vmask, V1.w & vmask};
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
 #pragma unroll
@@ -461,7 +453,7 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) l_run[nt][e] += __shfl_xor_sync(0xffffffffu, l_run[nt][e], o);
     const float unit = exp2i(-F);  // acc -> output units (|F| <= 125)
-    constexpr int kLd = kHeadDim + 1;
+    constexpr int kLd = kHeadDim + 4;    // padded rows: conflict-free stores, 16-byte aligned rows
     float* so = scratch;                 // [8*NT][kLd]
     float* sl = scratch + 8 * NT * kLd;  // [8*NT] base-2 lse
 #pragma unroll
@@ -487,7 +479,8 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
     __syncwarp();
     const int n_qv = NT == 1 ? g : n_members * g;
     for (int qv = 0; qv < n_qv; ++qv) {
-      const float o0 = so[qv * kLd + 2 * lane], o1 = so[qv * kLd + 2 * lane + 1];
+      const float2 o = *reinterpret_cast<const float2*>(so + qv * kLd + 2 * lane);
+      const float o0 = o.x, o1 = o.y;
       const float l2 = sl[qv];
       int tok, dst_slot;
       if (NT == 1) {
