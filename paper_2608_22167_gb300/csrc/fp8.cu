@@ -326,27 +326,32 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
           }
         }
 
-        float sv[NT][4];
+        // t = score - reference (base 2): one FFMA per score
+        float fk[NT][4], tv[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
-          sv[nt][0] = cc[nt][0] * (sc.x * qm[nt][0]);
-          sv[nt][1] = cc[nt][1] * (sc.x * qm[nt][1]);
-          sv[nt][2] = cc[nt][2] * (sc.y * qm[nt][0]);
-          sv[nt][3] = cc[nt][3] * (sc.y * qm[nt][1]);
+          fk[nt][0] = sc.x * qm[nt][0];
+          fk[nt][1] = sc.x * qm[nt][1];
+          fk[nt][2] = sc.y * qm[nt][0];
+          fk[nt][3] = sc.y * qm[nt][1];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) tv[nt][i] = fmaf(cc[nt][i], fk[nt][i], -m_ref[nt][i & 1]);
         }
         float u0 = sc.z, u1 = sc.w;
+        bool v0 = true, v1 = true;
         uint32_t vw[8] = {V0.x, V0.y, V0.z, V0.w, V1.x, V1.y, V1.z, V1.w};
         // a row's first and last pages may hold keys it does not see
         const int pk = (pb + k) * kPage;
         if (NT == 1 && (pk < first_key || pk + kPage > seq_len)) {
           const int klo = max(first_key - pk, 0), khi = min(seq_len - pk, kPage);
-          const bool v0 = key_a >= klo && key_a < khi, v1 = key_b >= klo && key_b < khi;
+          v0 = key_a >= klo && key_a < khi;
+          v1 = key_b >= klo && key_b < khi;
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            sv[nt][0] = v0 ? sv[nt][0] : -INFINITY;
-            sv[nt][1] = v0 ? sv[nt][1] : -INFINITY;
-            sv[nt][2] = v1 ? sv[nt][2] : -INFINITY;
-            sv[nt][3] = v1 ? sv[nt][3] : -INFINITY;
+            tv[nt][0] = v0 ? tv[nt][0] : -INFINITY;
+            tv[nt][1] = v0 ? tv[nt][1] : -INFINITY;
+            tv[nt][2] = v1 ? tv[nt][2] : -INFINITY;
+            tv[nt][3] = v1 ? tv[nt][3] : -INFINITY;
           }
           u0 = v0 ? u0 : 0.f;
           u1 = v1 ? u1 : 0.f;
@@ -360,8 +365,7 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
         bool over = fmaxf(u0, u1) >= u_lim;
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
-          over |= fmaxf(sv[nt][0], sv[nt][2]) > m_ref[nt][0] + kF8Lazy ||
-                  fmaxf(sv[nt][1], sv[nt][3]) > m_ref[nt][1] + kF8Lazy;
+          over |= fmaxf(fmaxf(tv[nt][0], tv[nt][2]), fmaxf(tv[nt][1], tv[nt][3])) > kF8Lazy;
         if (__any_sync(0xffffffffu, over)) {
           float um = fmaxf(u0, u1);
           um = fmaxf(um, __shfl_xor_sync(0xffffffffu, um, 4));
@@ -375,7 +379,11 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
           u_lim = exp2i(-F);
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            float mx0 = fmaxf(sv[nt][0], sv[nt][2]), mx1 = fmaxf(sv[nt][1], sv[nt][3]);
+            // exact scores again (the reference may still be the initial -1e30)
+            float sx[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) sx[i] = ((i < 2) ? v0 : v1) ? cc[nt][i] * fk[nt][i] : -INFINITY;
+            float mx0 = fmaxf(sx[0], sx[2]), mx1 = fmaxf(sx[1], sx[3]);
 #pragma unroll
             for (int o = 4; o < 32; o <<= 1) {
               mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
@@ -385,6 +393,8 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
             const float al0 = ex2_approx(m_ref[nt][0] - mn0), al1 = ex2_approx(m_ref[nt][1] - mn1);
             m_ref[nt][0] = mn0;
             m_ref[nt][1] = mn1;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) tv[nt][i] = sx[i] - m_ref[nt][i & 1];
             l_run[nt][0] *= al0;
             l_run[nt][1] *= al1;
             const float ac0 = al0 * dF, ac1 = al1 * dF;
@@ -402,8 +412,8 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
         uint32_t pv_hi[NT], pv_lo[NT];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
-          const float p00 = ex2_approx(sv[nt][0] - m_ref[nt][0]), p01 = ex2_approx(sv[nt][1] - m_ref[nt][1]);
-          const float p10 = ex2_approx(sv[nt][2] - m_ref[nt][0]), p11 = ex2_approx(sv[nt][3] - m_ref[nt][1]);
+          const float p00 = ex2_approx(tv[nt][0]), p01 = ex2_approx(tv[nt][1]);
+          const float p10 = ex2_approx(tv[nt][2]), p11 = ex2_approx(tv[nt][3]);
           l_run[nt][0] += p00 + p10;
           l_run[nt][1] += p01 + p11;
           // P' in fp16, split into e4m3 hi + lo; each key's (hi, lo) codes
