@@ -17,35 +17,28 @@
 // float arithmetic; an all-zero row stores zeros. A key is code * scale.
 //
 // Decode over fp8 pages follows the bf16 kernel (one warp per work item, a
-// per-warp ring of pages filled by one bulk copy each, online softmax in
-// fp32, partials merged by log-sum-exp) but multiplies on the fp8 tensor
-// cores (mma m16n8k32, e4m3 x e4m3 -> f32), so the codes go from shared
-// memory into the MMAs as they are:
-//   - S = K q: q (bf16) times a power of two per query vector (largest
-//     entry in [2^7, 2^8)) is split into two e4m3 pieces hi + mid. A bf16
-//     value has 8 significant bits, so hi (4 bits, nearest) leaves a
-//     residual that is an integer multiple of 2^-7 of the value's binade
-//     and at most 8 such units: mid holds it exactly unless it falls below
-//     the e4m3 subnormal quantum 2^-9 (entries under 2^-9 of the largest;
-//     their error is at most 2^-17 of it). The two pieces share one MMA
-//     through a duplicated K operand (4 MMAs per page). Each score is then
-//     scaled by its key's scale, the power of two and the softmax scale;
-//   - O += P' V: P' = p * v_scale * 2^F in fp16 (F a per-item power of two
-//     that only decreases, so that v_scale * 2^F < 1 and P' < 2^8) is
-//     split into e4m3 hi + lo, the
-//     two pieces sit in the two halves of the MMA's k range beside a
-//     duplicated V operand (4 MMAs per page). The accumulator is rescaled
-//     when F drops and divided by 2^F at the end.
-// Which keys meet in which MMA row/slot is a permutation chosen so that the
-// score fragment transposes into the P' operand with movmatrix: M row r of
-// the score tile is key 4(r/2) + (r%2), row r + 8 is that key + 2. The
-// running max is lazy: scores are exponentiated against a reference that
-// is only raised (with the rescale) when a score exceeds it by more than 8
-// (p <= 2^8), and F is only lowered when a page's V scale needs it; both
-// checks are one warp vote per page. On pages that a row sees only in part
-// (its first and last), V codes of invisible keys are zeroed in registers
-// (unwritten slots may hold any byte, e4m3 NaN included); a page outside
-// the pool is skipped.
+// per-warp ring of pages filled by one bulk copy each, m16n8k16 tensor-core
+// tiles, online softmax in fp32, partials merged by log-sum-exp):
+//   - codes become fp16 MMA operands by the hardware conversion of code
+//     pairs (exact: every e4m3 value is an fp16 value);
+//   - S = K q: q (bf16) enters as fp16 times a power of two per query
+//     vector (largest entry in [2^14, 2^15), exact for every bf16 entry
+//     above 2^-28 of it); each score is then scaled by its key's scale, the
+//     power of two and the softmax scale;
+//   - O += P' V: P' = p * v_scale * 2^F in fp16, F a per-item power of two
+//     that only decreases so that v_scale * 2^F < 1 and P' < 2^8; the
+//     accumulator is rescaled when F drops and divided by 2^F at the end.
+// MMA row r of the score tile is key 4(r/2) + (r%2) and row r + 8 is that
+// key + 2, so that movmatrix turns the score fragment into the P' operand
+// whose k-slots 2c, 2c + 1, 2c + 8, 2c + 9 are keys 4c .. 4c + 3, the keys
+// of one 32-bit word of V codes. The running max is lazy: scores are
+// exponentiated against a reference that is only raised (with the rescale)
+// when a score exceeds it by more than 8 (p <= 2^8), and F is only lowered
+// when a page's V scale needs it; both checks are one warp vote per page.
+// On pages that a row sees only in part (its first and last), codes of
+// invisible V slots are zeroed before conversion (unwritten slots may hold
+// any byte, e4m3 NaN included) and their scores masked; a page outside the
+// pool is skipped.
 #include <cuda_fp16.h>
 
 #include "common.cuh"
@@ -66,16 +59,6 @@ size_t decode_fp8_smem_bytes() {
   return 128 /* alignment slack */ + (size_t)kF8Warps * kF8RingBytes + (size_t)kF8Warps * kF8Stages * 8;
 }
 
-// D = A(16x32, row) * B(32x8, col) + D, e4m3 inputs, fp32 accumulators.
-__device__ __forceinline__ void mma_e4m3_16832(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                               uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
 // e4m3 codes of x0 (low byte) and x1 (high byte): nearest, ties to even,
 // saturating at +-448.
 __device__ __forceinline__ uint32_t e4m3x2(float x0, float x1) {
@@ -83,35 +66,18 @@ __device__ __forceinline__ uint32_t e4m3x2(float x0, float x1) {
   asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(d) : "f"(x1), "f"(x0));
   return d;
 }
-// the same from an f16 pair (low half -> low byte)
-__device__ __forceinline__ uint32_t e4m3x2_from_f16x2(uint32_t h) {
-  uint16_t d;
-  asm("cvt.rn.satfinite.e4m3x2.f16x2 %0, %1;" : "=h"(d) : "r"(h));
-  return d;
-}
-// exact f16 pair of two codes (low byte -> low half)
-__device__ __forceinline__ uint32_t f16x2_from_e4m3x2(uint32_t c) {
-  uint32_t h;
-  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h) : "h"((uint16_t)c));
-  return h;
-}
 __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
   __half2 v = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
-__device__ __forceinline__ uint32_t hsub2_u32(uint32_t a, uint32_t b) {
-  __half2 r = __hsub2(*reinterpret_cast<__half2*>(&a), *reinterpret_cast<__half2*>(&b));
-  return *reinterpret_cast<uint32_t*>(&r);
-}
-__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
-  uint32_t d;
-  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
-  return d;
-}
-// value of each code of a pair, as floats
-__device__ __forceinline__ float2 e4m3x2_value(uint32_t c) {
-  const uint32_t h = f16x2_from_e4m3x2(c);
-  return __half22float2(*reinterpret_cast<const __half2*>(&h));
+// the four codes of a word as two exact f16 pairs: (bytes 0, 1) and (2, 3)
+__device__ __forceinline__ void f16x2x2_from_e4m3x4(uint32_t w, uint32_t& lo, uint32_t& hi) {
+  asm("{\n\t.reg .b16 l16, h16;\n\t"
+      "mov.b32 {l16, h16}, %2;\n\t"
+      "cvt.rn.f16x2.e4m3x2 %0, l16;\n\t"
+      "cvt.rn.f16x2.e4m3x2 %1, h16;\n\t}"
+      : "=r"(lo), "=r"(hi)
+      : "r"(w));
 }
 
 // 2^e as a float for -126 <= e <= 127
@@ -129,8 +95,8 @@ __device__ __forceinline__ uint32_t key_byte_mask(int c, int lo, int hi) {
 }
 
 template <int NT>
-__global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_kernel(const uint8_t* __restrict__ kv8,
-                                                                   const AttnParams p) {
+__global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1)
+    decode_fp8_kernel(const uint8_t* __restrict__ kv8, const AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
@@ -189,10 +155,10 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
     }
     const int* bt_row = p.block_table + (size_t)row * p.max_pages;
 
-    // Query vector r (+ 8 nt) as B operands: this lane holds its dims
-    // 16c .. 16c + 15 as e4m3 pieces of q * 2^eq. MMA step j takes dims
-    // 16c + 4j .. + 3, hi in k-slots 0..15 and mid in 16..31.
-    uint32_t q_hi[NT][4], q_mid[NT][4];
+    // Query vector r (+ 8 nt) as the B operand: this lane holds its dims
+    // 16c .. 16c + 15 as fp16 of q * 2^eq; MMA step kk takes dims
+    // 16c + 4kk, +1 (k-slots 2c, 2c + 1) and 16c + 4kk + 2, +3 (2c + 8, 2c + 9).
+    uint32_t qb[NT][4][2];
     float qm[NT][2];  // score factor of query vectors 2c and 2c + 1
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
@@ -223,22 +189,13 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
       for (int i = 0; i < 16; ++i) mx = fmaxf(mx, fabsf(x[i]));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      int eq = mx > 0.f ? 7 - ilog2f(mx) : 0;
+      int eq = mx > 0.f ? 14 - ilog2f(mx) : 0;
       eq = min(max(eq, -126), 126);
       const float up = exp2i(eq);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {  // word j: dims 16c + 4j .. + 3
-        uint32_t h = 0, m = 0;
-#pragma unroll
-        for (int i = 0; i < 4; i += 2) {
-          const float a0 = x[4 * j + i] * up, a1 = x[4 * j + i + 1] * up;
-          const uint32_t ch = e4m3x2(a0, a1);
-          const float2 vh = e4m3x2_value(ch);
-          h |= ch << (8 * i);
-          m |= e4m3x2(a0 - vh.x, a1 - vh.y) << (8 * i);  // the residuals are exact in float
-        }
-        q_hi[nt][j] = h;
-        q_mid[nt][j] = m;
+      for (int kk = 0; kk < 4; ++kk) {
+        qb[nt][kk][0] = pack_f16x2(x[4 * kk] * up, x[4 * kk + 1] * up);
+        qb[nt][kk][1] = pack_f16x2(x[4 * kk + 2] * up, x[4 * kk + 3] * up);
       }
       const float my_qm = exp2i(-eq) * p.scale_log2;
       qm[nt][0] = __shfl_sync(0xffffffffu, my_qm, (2 * c) * 4);
@@ -320,9 +277,12 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
         {
           const uint32_t wa[4] = {KA.x, KA.y, KA.z, KA.w}, wb[4] = {KB.x, KB.y, KB.z, KB.w};
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
+          for (int kk = 0; kk < 4; ++kk) {
+            uint32_t a0, a1, a2, a3;
+            f16x2x2_from_e4m3x4(wa[kk], a0, a2);
+            f16x2x2_from_e4m3x4(wb[kk], a1, a3);
 #pragma unroll
-            for (int j = 0; j < 4; ++j) mma_e4m3_16832(cc[nt], wa[j], wb[j], wa[j], wb[j], q_hi[nt][j], q_mid[nt][j]);
+            for (int nt = 0; nt < NT; ++nt) mma_f16_16816(cc[nt], a0, a1, a2, a3, qb[nt][kk][0], qb[nt][kk][1]);
           }
         }
 
@@ -409,34 +369,25 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1) decode_fp8_ker
         }
         const float w0 = u0 * pf, w1 = u1 * pf;
 
-        uint32_t pv_hi[NT], pv_lo[NT];
+        uint32_t pb0[NT], pb1[NT];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
           const float p00 = ex2_approx(tv[nt][0]), p01 = ex2_approx(tv[nt][1]);
           const float p10 = ex2_approx(tv[nt][2]), p11 = ex2_approx(tv[nt][3]);
           l_run[nt][0] += p00 + p10;
           l_run[nt][1] += p01 + p11;
-          // P' in fp16, split into e4m3 hi + lo; each key's (hi, lo) codes
-          // form one 16-bit element for the transpose
-          const uint32_t fa = pack_f16x2(p00 * w0, p01 * w0), fb = pack_f16x2(p10 * w1, p11 * w1);
-          const uint32_t ha = e4m3x2_from_f16x2(fa), hb = e4m3x2_from_f16x2(fb);
-          const uint32_t la = e4m3x2_from_f16x2(hsub2_u32(fa, f16x2_from_e4m3x2(ha)));
-          const uint32_t lb = e4m3x2_from_f16x2(hsub2_u32(fb, f16x2_from_e4m3x2(hb)));
-          const uint32_t t0 = movmatrix_trans(prmt(ha, la, 0x5140u));  // keys 4c, 4c + 1 of column r
-          const uint32_t t1 = movmatrix_trans(prmt(hb, lb, 0x5140u));  // keys 4c + 2, 4c + 3
-          pv_hi[nt] = prmt(t0, t1, 0x6420u);
-          pv_lo[nt] = prmt(t0, t1, 0x7531u);
+          pb0[nt] = movmatrix_trans(pack_f16x2(p00 * w0, p01 * w0));  // keys 4c, 4c + 1 of column r
+          pb1[nt] = movmatrix_trans(pack_f16x2(p10 * w1, p11 * w1));  // keys 4c + 2, 4c + 3
         }
 
-        // O^T[64 dims x 8*NT] += V^T P'^T: k-slots 0..15 carry the hi piece,
-        // 16..31 the lo piece, both against the same V codes (dims
-        // 16 mt + r and 16 mt + 8 + r, keys 4c .. 4c + 3)
+        // O^T[64 dims x 8*NT] += V^T P'^T over dims 16 mt + r and 16 mt + 8 + r
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
+          uint32_t a0, a1, a2, a3;
+          f16x2x2_from_e4m3x4(vw[2 * mt], a0, a2);
+          f16x2x2_from_e4m3x4(vw[2 * mt + 1], a1, a3);
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
-            mma_e4m3_16832(acc[mt][nt], vw[2 * mt], vw[2 * mt + 1], vw[2 * mt], vw[2 * mt + 1], pv_hi[nt],
-                           pv_lo[nt]);
+          for (int nt = 0; nt < NT; ++nt) mma_f16_16816(acc[mt][nt], a0, a1, a2, a3, pb0[nt], pb1[nt]);
         }
       }
 
