@@ -8,8 +8,9 @@
 //     per-warp ring of NSTAGE stages filled by 2-D TMA loads (128-byte
 //     swizzle, so ldmatrix reads are bank-conflict free);
 //   - computes S^T = K Q^T with mma.sync m16n8k16 (16 keys as M, query
-//     vectors as N), applies the causal/window/length mask and an online
-//     softmax in fp32 (base-2 exponent, scale folded in);
+//     vectors as N), masks keys outside [first_key, seq_len) on a row's
+//     first and last page, and runs an online softmax in fp32 (base-2
+//     exponent, scale folded in) against a lazily raised reference max;
 //   - transposes P^T into the B operand with movmatrix and accumulates
 //     O^T += V^T P^T (head dim as M) in fp32.
 // The item ends with either the final bf16 output + lse (a decode row that
@@ -153,10 +154,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     const int pre = n < kDecodeStages ? n : kDecodeStages;
     for (int k = 0; k < pre; ++k) issue(k);
 
-    float m_run[NT][2], l_run[NT][2], acc[4][NT][4];
+    // Online softmax with a lazy reference: scores are exponentiated against
+    // m_ref, which is only raised (with the rescale of O and l) when a score
+    // exceeds it by more than kLazy (so p <= 2^8, exact enough in bf16);
+    // checking that is one warp vote per page.
+    constexpr float kLazy = 8.f;
+    constexpr float kNoMax = -1e30f;  // reference before the first visible key
+    float m_ref[NT][2], l_run[NT][2], acc[4][NT][4];
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
-      m_run[nt][0] = m_run[nt][1] = -INFINITY;
+      m_ref[nt][0] = m_ref[nt][1] = kNoMax;
       l_run[nt][0] = l_run[nt][1] = 0.f;
 #pragma unroll
       for (int mt = 0; mt < 4; ++mt)
@@ -187,43 +194,65 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(c[nt], a0, a1, a2, a3, qb[nt][kk][0], qb[nt][kk][1]);
       }
 
-      // mask keys outside [first_key, seq_len) (partial first/last page)
+      // t = score - reference (base 2), one FFMA each
+      float tv[NT][4];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) tv[nt][i] = fmaf(c[nt][i], p.scale_log2, -m_ref[nt][i & 1]);
+      // keys outside [first_key, seq_len): only a row's first and last pages
       const int j0 = (pb + k) * kPage + (lane >> 2);
       bool v0 = true, v1 = true;
-      if (NT == 1) {
+      if (NT == 1 && ((pb + k) * kPage < first_key || (pb + k + 1) * kPage > seq_len)) {
         v0 = j0 >= first_key && j0 < seq_len;
         v1 = (j0 + 8) >= first_key && (j0 + 8) < seq_len;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          tv[nt][0] = v0 ? tv[nt][0] : -INFINITY;
+          tv[nt][1] = v0 ? tv[nt][1] : -INFINITY;
+          tv[nt][2] = v1 ? tv[nt][2] : -INFINITY;
+          tv[nt][3] = v1 ? tv[nt][3] : -INFINITY;
+        }
+      }
+      bool over = false;
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) over |= fmaxf(fmaxf(tv[nt][0], tv[nt][2]), fmaxf(tv[nt][1], tv[nt][3])) > kLazy;
+      if (__any_sync(0xffffffffu, over)) {  // rare: raise the reference to the running max
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          float sx[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) sx[i] = ((i < 2) ? v0 : v1) ? c[nt][i] * p.scale_log2 : -INFINITY;
+          float mx0 = fmaxf(sx[0], sx[2]), mx1 = fmaxf(sx[1], sx[3]);
+#pragma unroll
+          for (int o = 4; o < 32; o <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+          }
+          const float mn0 = fmaxf(m_ref[nt][0], mx0), mn1 = fmaxf(m_ref[nt][1], mx1);
+          const float al0 = ex2_approx(m_ref[nt][0] - mn0), al1 = ex2_approx(m_ref[nt][1] - mn1);
+          m_ref[nt][0] = mn0;
+          m_ref[nt][1] = mn1;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) tv[nt][i] = sx[i] - m_ref[nt][i & 1];
+          l_run[nt][0] *= al0;
+          l_run[nt][1] *= al1;
+#pragma unroll
+          for (int mt = 0; mt < 4; ++mt) {
+            acc[mt][nt][0] *= al0;
+            acc[mt][nt][1] *= al1;
+            acc[mt][nt][2] *= al0;
+            acc[mt][nt][3] *= al1;
+          }
+        }
       }
       uint32_t pb0[NT], pb1[NT];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        const float s00 = v0 ? c[nt][0] * p.scale_log2 : -INFINITY;
-        const float s01 = v0 ? c[nt][1] * p.scale_log2 : -INFINITY;
-        const float s10 = v1 ? c[nt][2] * p.scale_log2 : -INFINITY;
-        const float s11 = v1 ? c[nt][3] * p.scale_log2 : -INFINITY;
-        float mx0 = fmaxf(s00, s10), mx1 = fmaxf(s01, s11);
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-          mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-          mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-        }
-        const float mn0 = fmaxf(m_run[nt][0], mx0), mn1 = fmaxf(m_run[nt][1], mx1);
-        const float mu0 = mn0 == -INFINITY ? 0.f : mn0;
-        const float mu1 = mn1 == -INFINITY ? 0.f : mn1;
-        const float al0 = fast_exp2(m_run[nt][0] - mu0), al1 = fast_exp2(m_run[nt][1] - mu1);
-        const float p00 = fast_exp2(s00 - mu0), p10 = fast_exp2(s10 - mu0);
-        const float p01 = fast_exp2(s01 - mu1), p11 = fast_exp2(s11 - mu1);
-        l_run[nt][0] = l_run[nt][0] * al0 + p00 + p10;
-        l_run[nt][1] = l_run[nt][1] * al1 + p01 + p11;
-        m_run[nt][0] = mn0;
-        m_run[nt][1] = mn1;
-#pragma unroll
-        for (int mt = 0; mt < 4; ++mt) {
-          acc[mt][nt][0] *= al0;
-          acc[mt][nt][1] *= al1;
-          acc[mt][nt][2] *= al0;
-          acc[mt][nt][3] *= al1;
-        }
+        const float p00 = ex2_approx(tv[nt][0]), p01 = ex2_approx(tv[nt][1]);
+        const float p10 = ex2_approx(tv[nt][2]), p11 = ex2_approx(tv[nt][3]);
+        l_run[nt][0] += p00 + p10;
+        l_run[nt][1] += p01 + p11;
         pb0[nt] = movmatrix_trans(pack_bf16x2(p00, p01));
         pb1[nt] = movmatrix_trans(pack_bf16x2(p10, p11));
       }
@@ -242,7 +271,6 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
       __syncwarp();
       if (k + kDecodeStages < n) issue(k + kDecodeStages);
     }
-
     if (timed_out) {
       raise_status(p, kStatusTimeout);
       return;  // the ring's phase tracking is lost: this warp stops here
@@ -265,11 +293,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
       for (int e = 0; e < 2; ++e) {
         const int qv = nt * 8 + 2 * (lane & 3) + e;
         const float l = l_run[nt][e];
+        const float m = l > 0.f ? m_ref[nt][e] : -INFINITY;
         float inv = l > 0.f ? 1.f / l : 0.f;
-        float lse2 = l > 0.f ? m_run[nt][e] + __log2f(l) : -INFINITY;
+        float lse2 = l > 0.f ? m + __log2f(l) : -INFINITY;
         // a row finished here (one split) takes its sink now; split rows in the merge
         if (NT == 1 && p.sinks != nullptr && slot < 0 && qv < g)
-          inv = finish_with_sink(m_run[nt][e], l, sink_log2(p, kvh * g + qv), &lse2);
+          inv = finish_with_sink(m, l, sink_log2(p, kvh * g + qv), &lse2);
 #pragma unroll
         for (int mt = 0; mt < 4; ++mt) {
           so[qv * kLd + mt * 16 + (lane >> 2)] = acc[mt][nt][e] * inv;
