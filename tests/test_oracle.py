@@ -709,3 +709,57 @@ def test_sampled_fp8_evaluation_equals_full_evaluation():
     heads = rng.integers(0, h["q"].shape[1], size=24).astype(np.int32)
     so, sl = oracle.paged_attention_sampled_fp8(h["q"], k8, v8, ks, vs, *args, toks, heads)
     assert np.array_equal(so, out[toks, heads]) and np.array_equal(sl, lse[toks, heads])
+
+
+def _quantize_pool_oracle(k_bits, v_bits):
+    """Whole bf16 pools quantized by the oracle (each page appended as one 16-token row)."""
+    P, H, page, D = k_bits.shape
+    tok = lambda x: np.ascontiguousarray(x.transpose(0, 2, 1, 3).reshape(P * page, H, D))  # noqa: E731
+    z8 = np.zeros((P, H, page, D), np.uint8)
+    zs = np.zeros((P, H, page), np.float32)
+    return oracle.kv_append_fp8(tok(k_bits), tok(v_bits), z8, z8, zs, zs, np.arange(P, dtype=np.int32)[:, None],
+                                np.full(P, page, np.int32), np.arange(P + 1, dtype=np.int32) * page)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_fp8_storage_error_stays_within_its_bounds(seed):
+    # What the fp8 format changes against bf16 attention on the same inputs:
+    # with every score moved by at most delta (sup norm), lse moves by at most
+    # delta (log-sum-exp is 1-Lipschitz in the sup norm) and every softmax
+    # weight by a factor within e^(+-2 delta), so
+    #   |out8 - out16| <= max_j |V8_j - V16_j| + (e^(2 delta) - 1) max_j |V16_j|
+    # per output dim, plus the final bf16 rounding of both outputs.
+    b = W.fuzz_batch(700 + seed)
+    h = W.host_inputs(b)
+    kc, vc = oracle.kv_append(h["k_new"], h["v_new"], h["k_cache"], h["v_cache"], h["block_table"],
+                              h["seq_lens"], h["query_start_loc"])
+    k8, v8, ks, vs = _quantize_pool_oracle(kc, vc)
+    args = (h["block_table"], h["seq_lens"], h["query_start_loc"], h["sliding_window"], h["softmax_scale"])
+    o16, l16 = oracle.paged_attention(h["q"], kc, vc, *args)
+    o8, l8 = oracle.paged_attention_fp8(h["q"], k8, v8, ks, vs, *args)
+    val = np.array([oracle.e4m3_to_float(c) for c in range(256)])
+    kd, vd = val[k8] * ks[..., None], val[v8] * vs[..., None]  # dequantized pools
+    kf, vf = _f(kc), _f(vc)
+    q = _f(h["q"])
+    g = b.num_q_heads // b.num_kv_heads
+    qsl, sl, bt = h["query_start_loc"], h["seq_lens"], h["block_table"]
+    checked = 0
+    for r in range(len(sl)):
+        S, L = int(sl[r]), int(qsl[r + 1] - qsl[r])
+        for i in range(L):
+            t, pos = int(qsl[r]) + i, S - L + i
+            lo = 0 if h["sliding_window"] <= 0 else max(0, pos - h["sliding_window"] + 1)
+            js = np.arange(lo, pos + 1)
+            pg, sl_ = bt[r, js // 16], js % 16
+            for hq in range(b.num_q_heads):
+                kv = hq // g
+                dk = kd[pg, kv, sl_] - kf[pg, kv, sl_]
+                delta = h["softmax_scale"] * np.max(np.abs(dk @ q[t, hq]))
+                assert abs(float(l8[t, hq]) - float(l16[t, hq])) <= delta + 1e-5
+                dv = np.max(np.abs(vd[pg, kv, sl_] - vf[pg, kv, sl_]), axis=0)
+                vmax = np.max(np.abs(vf[pg, kv, sl_]), axis=0)
+                bound = dv + np.expm1(2 * delta) * vmax
+                ref = _f(o16[t, hq])
+                assert np.all(np.abs(_f(o8[t, hq]) - ref) <= bound + 2.0**-8 * (np.abs(ref) + bound) + 1e-30)
+                checked += 1
+    assert checked > 0
