@@ -94,6 +94,7 @@ FP8_SOURCES = [
     "paper_2608_22167_gb300/csrc/common.cuh",
 ]
 FP8_WORKLOADS = ("tiny", "decode", "long")
+NOMINAL_HBM_GBS = 8000.0  # the nominal HBM3e figure the targets are also quoted against
 
 
 def peaks():
@@ -365,6 +366,26 @@ def oracle_fp8_pools(k_bits, v_bits):
                                 np.full(P, page, np.int32), np.arange(P + 1, dtype=np.int32) * page)
 
 
+def cpu_model() -> str:
+    """The host CPU's name (x86 'model name', else the Arm implementer/part)."""
+    try:
+        info = open("/proc/cpuinfo").read()
+    except OSError:
+        return "unknown"
+    for line in info.splitlines():
+        if line.lower().startswith("model name"):
+            return line.split(":", 1)[1].strip()
+    parts = {"0x41": "Arm", "0x4e": "NVIDIA"}
+    impl = part = None
+    for line in info.splitlines():
+        if line.startswith("CPU implementer") and impl is None:
+            impl = line.split(":", 1)[1].strip()
+        if line.startswith("CPU part") and part is None:
+            part = line.split(":", 1)[1].strip()
+    names = {"0xd4f": "Neoverse-V2"}
+    return f"{parts.get(impl, impl)} {names.get(part, part)}" if impl else "unknown"
+
+
 def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int, kv: str = "bf16"):
     """Time the oracle on a bounded sample of the workload and scale its
     throughput to the whole step by attended (query, key) pairs."""
@@ -424,6 +445,7 @@ def cpu_baseline_sample(batch: W.Batch, stats_total, seconds: float, seed: int, 
         value=stats_total["kv_bytes"] / est_step_s / 1e9,
         unit="GB/s",
         cores=int(oracle.max_threads()),
+        cpu_model=cpu_model(),
         kind="oracle",
         sample=f"{'fp8 pages, ' if kv == 'fp8' else ''}"
                f"{n_tok} query tokens x {batch.num_q_heads} heads from {rounds} draws of 6 decode + 2 append "
@@ -540,10 +562,12 @@ def run_ours(args, rank, world, dev):
     # decode, [2]->[3] cascade (side stream), [1]->[4] append; the merge
     # starts at the join, the later of [3] and [4].
     ktime = {n: 0.0 for n in ("plan", "decode", "cascade", "append_chunk", "merge")}
+    layer_ms = [0.0] * nl  # each layer's forward span (planner to merge)
     for k in range(n_sets):
         for i in range(nl):
             ev = phase[k][i]
             t = [0.0] + [ev[0].elapsed_time(ev[j]) for j in range(1, len(ev))]
+            layer_ms[i] += t[5] / n_sets
             ktime["plan"] += t[1]
             ktime["decode"] += t[2] - t[1]
             ktime["cascade"] += t[3] - t[2]
@@ -637,6 +661,12 @@ def run_ours(args, rank, world, dev):
     # ---- max over ranks
     total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], dev, world)
     ms_per_step = total_ms / args.steps
+    # the step's own bound: max(KV bytes / HBM peak, attention flops / bf16 peak)
+    flops = sum(s["flops"] for s in per_layer)
+    ideal_ms = max(kv_bytes / (hbm * 1e9), flops / (tc_burst * 1e12)) * 1e3
+    combined = {"ideal_ms": round(ideal_ms, 4), "frac": round(ideal_ms / ms_per_step, 4),
+                "bound": "hbm" if kv_bytes / (hbm * 1e9) >= flops / (tc_burst * 1e12) else "tensor",
+                "flops_per_step": int(flops)}
     value = whole_job_gbs(kv_bytes, world, ms_per_step)
     e2e_value = whole_job_gbs(kv_bytes, world, e2e_ms)
 
@@ -663,14 +693,18 @@ def run_ours(args, rank, world, dev):
             "kv_bytes_per_step": kv_bytes,
             "attended_pairs_per_step": pairs,
             "l2": "inputs larger than L2 (KV pool %.1f GB >> 126 MB L2); no flush" % (
-                sum(p.k_cache.numel() * 4 for p in batch.pools.values()) / 1e9),
+                sum(p.k_cache.numel() * (4 if not fp8 else 2 * (batch.head_dim + 4) / batch.head_dim)
+                    for p in batch.pools.values()) / 1e9),
             "parallelism": f"replicas x{world} (no exchange step)",
             "launch": "one CUDA graph per step (KV append + forward of every layer)" if graphs
                       else "eager (C-ABI calls per layer)",
         },
         "frac_of_hbm_peak": round(value / world / hbm, 4),
+        "frac_of_nominal_hbm": round(value / world / NOMINAL_HBM_GBS, 4),
+        "combined_roofline": combined,
         "attended_tokens_per_s": round(pairs * world / (ms_per_step * 1e-3), 1),
         "kernel_ms_per_step": {k: round(v, 4) for k, v in ktime.items()},
+        "layer_ms": [round(v, 4) for v in layer_ms] if nl > 1 else None,
         ("eager_ms_per_step" if graphs else "graph_ms_per_step"): (round(other_ms, 4) if other_ms else None),
         "roofline": dominant,
         "roofline_decode": roof_dec,
@@ -853,8 +887,8 @@ def run_reference(args, rank, world):
         "config": {"workload": ("fp8 KV pages, " if args.kv == "fp8" else "") + WORKLOAD_DESC[args.workload],
                    "kv": args.kv, "layers": nl, "rows": batch.num_seqs},
         "impl": "reference",
-        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cb["cores"], "kind": "oracle",
-                         "sample": cb["sample"]},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cb["cores"],
+                         "cpu_model": cb["cpu_model"], "kind": "oracle", "sample": cb["sample"]},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
