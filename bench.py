@@ -102,7 +102,8 @@ def peaks():
     try:
         with open(path) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured"
+        sustained = float(d.get("bf16_tflops_sustained", d["bf16_tflops"]))
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), sustained, "measured"
     except Exception:
         return 6800.0, 1900.0, 1700.0, "fallback"
 
@@ -332,7 +333,8 @@ class Fp8Stepper(Stepper):
         super().__init__(batch, dev)
         self.pools8 = quantize_pools_fp8(batch, dev)
         for i, lay in enumerate(batch.layers):
-            self.launches_per_layer[i] = 4 + (1 if lay.sliding_window <= 0 else 0)  # append, plan, decode, [cascade], merge
+            # append, plan, decode, [cascade], merge
+            self.launches_per_layer[i] = 4 + (1 if lay.sliding_window <= 0 else 0)
 
     def layer_call(self, i, q=None, k_new=None, v_new=None, out=None, lse=None, events=None):
         m = self.mcpu
