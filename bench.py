@@ -275,7 +275,8 @@ class Stepper:
         self.launches_per_layer = {}
         for i, lay in enumerate(batch.layers):
             cascade = 1 if lay.sliding_window <= 0 else 0
-            self.launches_per_layer[i] = 5 + cascade  # append, plan, [cascade], decode, append-chunk, merge
+            # KV append, [prefix scan], plan, decode, [cascade], append chunks, merge
+            self.launches_per_layer[i] = 5 + 2 * cascade
 
     def layer_call(self, i, q=None, k_new=None, v_new=None, out=None, lse=None, events=None):
         m = self.mcpu
@@ -333,8 +334,8 @@ class Fp8Stepper(Stepper):
         super().__init__(batch, dev)
         self.pools8 = quantize_pools_fp8(batch, dev)
         for i, lay in enumerate(batch.layers):
-            # append, plan, decode, [cascade], merge
-            self.launches_per_layer[i] = 4 + (1 if lay.sliding_window <= 0 else 0)
+            # KV append, [prefix scan], plan, decode, [cascade], merge
+            self.launches_per_layer[i] = 4 + 2 * (1 if lay.sliding_window <= 0 else 0)
 
     def layer_call(self, i, q=None, k_new=None, v_new=None, out=None, lse=None, events=None):
         m = self.mcpu
@@ -565,11 +566,14 @@ def run_ours(args, rank, world, dev):
     # starts at the join, the later of [3] and [4].
     ktime = {n: 0.0 for n in ("plan", "decode", "cascade", "append_chunk", "merge")}
     layer_ms = [0.0] * nl  # each layer's forward span (planner to merge)
+    layer_k = [[0.0] * 5 for _ in range(nl)]  # plan, decode+cascade, append, merge (from the join), total
     for k in range(n_sets):
         for i in range(nl):
             ev = phase[k][i]
             t = [0.0] + [ev[0].elapsed_time(ev[j]) for j in range(1, len(ev))]
             layer_ms[i] += t[5] / n_sets
+            for j, v in enumerate((t[1], t[3] - t[1], t[4] - t[1], t[5] - max(t[3], t[4]), t[5])):
+                layer_k[i][j] += v / n_sets
             ktime["plan"] += t[1]
             ktime["decode"] += t[2] - t[1]
             ktime["cascade"] += t[3] - t[2]
@@ -707,6 +711,8 @@ def run_ours(args, rank, world, dev):
         "attended_tokens_per_s": round(pairs * world / (ms_per_step * 1e-3), 1),
         "kernel_ms_per_step": {k: round(v, 4) for k, v in ktime.items()},
         "layer_ms": [round(v, 4) for v in layer_ms] if nl > 1 else None,
+        "layer_kernel_ms": ({"plan, decode+cascade, append, merge, total": [
+            [round(v, 4) for v in layer_k[i]] for i in range(min(nl, 2))]} if nl > 1 else None),
         ("eager_ms_per_step" if graphs else "graph_ms_per_step"): (round(other_ms, 4) if other_ms else None),
         "roofline": dominant,
         "roofline_decode": roof_dec,

@@ -78,6 +78,7 @@ static_assert(sizeof(PlanHeader) == 256, "header is one 256-byte block");
 // Byte offsets of every array inside the workspace, derived from the dims.
 struct WorkspaceLayout {
   size_t header, decode_items, cascade_items, members, append_items, merge_rows;
+  size_t lcp;  // per row: leading physical pages equal to the previous row's (shared-prefix scan)
   size_t o_part, lse_part, total;
   int32_t max_decode, max_cascade, max_append, max_parts;
 };
@@ -99,6 +100,7 @@ __host__ __device__ inline WorkspaceLayout workspace_layout(int32_t num_seqs, in
   w.members = off;       off = align_up(off + sizeof(CascadeMember) * (size_t)(num_seqs + 1), 256);
   w.append_items = off;  off = align_up(off + sizeof(AppendItem) * (size_t)w.max_append, 256);
   w.merge_rows = off;    off = align_up(off + sizeof(MergeRow) * (size_t)(num_seqs + 1), 256);
+  w.lcp = off;           off = align_up(off + sizeof(int32_t) * (size_t)(num_seqs + 1), 256);
   w.o_part = off;        off = align_up(off + sizeof(float) * (size_t)w.max_parts * num_q_heads * kHeadDim, 256);
   w.lse_part = off;      off = align_up(off + sizeof(float) * (size_t)w.max_parts * num_q_heads, 256);
   w.total = off;

@@ -176,68 +176,13 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
 
   // ---- phase 2: shared-prefix groups (full-context calls only)
   // lcp[r] = leading physical pages row r shares with row r - 1 (full pages
-  // of both). First the leading kLcpProbe pages of every adjacent pair are
-  // compared by all threads at once (most pairs differ at once, group
-  // members agree over the probe); pairs that agree over the whole probe go
-  // on warp by warp, 128 entries per step.
-  constexpr int kLcpProbe = 32;
+  // of both), scanned beforehand by lcp_kernel across the whole GPU.
   const bool cascade = p.cascade_enabled && p.window <= 0;
   if (cascade) {
+    const int* lcp_ws = reinterpret_cast<const int*>(p.ws + p.lay.lcp);
     for (int r = tid; r < B; r += NT) {
       const int sa = r > 0 ? sm.S[r - 1] : -1, sb = sm.S[r];
-      sm.lcp[r] = (sa < 0 || sb < 0) ? 0 : min(min(sa, sb) / kPage, kLcpProbe);
-    }
-    __syncthreads();
-    // four compares per thread in flight: all loads first, then the checks
-    const int n_cmp = (B - 1) * kLcpProbe;
-    for (int e0 = tid; e0 < n_cmp; e0 += 4 * NT) {
-      int va[4], vb[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int e = e0 + j * NT, r = 1 + e / kLcpProbe, i = e % kLcpProbe;
-        const bool in = e < n_cmp && i < p.max_pages;
-        va[j] = in ? __ldg(p.block_table + (size_t)(r - 1) * p.max_pages + i) : 0;
-        vb[j] = in ? __ldg(p.block_table + (size_t)r * p.max_pages + i) : 0;
-      }
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int e = e0 + j * NT, r = 1 + e / kLcpProbe, i = e % kLcpProbe;
-        if (e < n_cmp && va[j] != vb[j] && i < sm.lcp[r]) atomicMin(&sm.lcp[r], i);
-      }
-    }
-    __syncthreads();
-    for (int r = warp + 1; r < B; r += kWarps) {
-      const int sa = sm.S[r - 1], sb = sm.S[r];
-      if (sa < 0 || sb < 0 || sm.lcp[r] < kLcpProbe) continue;
-      const int lim = min(sa, sb) / kPage;  // pages full in both rows
-      const int* ba = p.block_table + (size_t)(r - 1) * p.max_pages;
-      const int* bb = p.block_table + (size_t)r * p.max_pages;
-      // 128 entries per step: four independent loads per lane, then ballots
-      int n = kLcpProbe;
-      for (int base = kLcpProbe; base < lim; base += 128) {
-        bool eq[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int i = base + 32 * j + lane;
-          eq[j] = i < lim && __ldg(ba + i) == __ldg(bb + i);
-        }
-        bool stop = false;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const unsigned m = __ballot_sync(0xffffffffu, eq[j]);
-          if (!stop) {
-            if (m == 0xffffffffu) {
-              n += 32;
-            } else {
-              n += __ffs(~m) - 1;
-              stop = true;
-            }
-          }
-        }
-        if (stop) break;
-      }
-      __syncwarp();
-      if (lane == 0) sm.lcp[r] = min(n, lim);
+      sm.lcp[r] = (sa < 0 || sb < 0) ? 0 : min(lcp_ws[r], min(sa, sb) / kPage);
     }
   }
   __syncthreads();
@@ -469,8 +414,61 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
   }
 }
 
+// One warp per adjacent row pair (r - 1, r): the number of leading block-table
+// entries the two rows share, over the pages full in both (lengths outside
+// the table count as none). 512 entries per step: 16 loads of each row per
+// lane in flight, one ballot per 32. Writes lcp[r] (lcp[0] = 0).
+constexpr int kLcpWarps = 8;
+constexpr int kLcpPerLane = 16;
+
+__global__ void __launch_bounds__(kLcpWarps * 32) lcp_kernel(const AttnParams p) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * kLcpWarps + (threadIdx.x >> 5);
+  int* lcp = reinterpret_cast<int*>(p.ws + p.lay.lcp);
+  if (r >= p.num_seqs) return;
+  if (r == 0) {
+    if (lane == 0) lcp[0] = 0;
+    return;
+  }
+  const int cap = p.max_pages * kPage;
+  const int sa = __ldg(p.seq_lens + r - 1), sb = __ldg(p.seq_lens + r);
+  const int lim = (sa < 0 || sb < 0 || sa > cap || sb > cap) ? 0 : min(sa, sb) / kPage;
+  const int* ba = p.block_table + (size_t)(r - 1) * p.max_pages;
+  const int* bb = p.block_table + (size_t)r * p.max_pages;
+  int n = 0;
+  for (int base = 0; base < lim; base += 32 * kLcpPerLane) {
+    int va[kLcpPerLane], vb[kLcpPerLane];
+#pragma unroll
+    for (int j = 0; j < kLcpPerLane; ++j) {
+      const int i = base + 32 * j + lane;
+      va[j] = i < lim ? __ldg(ba + i) : 0;
+      vb[j] = i < lim ? __ldg(bb + i) : 1;
+    }
+    bool stop = false;
+#pragma unroll
+    for (int j = 0; j < kLcpPerLane; ++j) {
+      const unsigned m = __ballot_sync(0xffffffffu, va[j] == vb[j]);
+      if (!stop) {
+        if (m == 0xffffffffu) {
+          n += 32;
+        } else {
+          n += __ffs(~m) - 1;
+          stop = true;
+        }
+      }
+    }
+    if (stop) break;
+  }
+  if (lane == 0) lcp[r] = min(n, lim);
+}
+
 cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream) {
   static_assert(sizeof(PlanSmem) < 200 * 1024, "planner shared memory");
+  if (p.cascade_enabled && p.window <= 0 && p.num_seqs > 0) {
+    lcp_kernel<<<(p.num_seqs + kLcpWarps - 1) / kLcpWarps, kLcpWarps * 32, 0, stream>>>(p);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   // fewer threads for small batches: every phase ends in a CTA barrier, and
   // barriers over 8 warps are cheaper than over 32
   if (p.num_seqs <= R * 256)
