@@ -148,6 +148,40 @@ def test_groups_larger_than_a_cascade_item():
     assert run.header()["n_cascade"] >= 2
 
 
+def _ws_lcp_offset(B, T, g):
+    """Byte offset of the per-row shared-prefix array in the workspace (the
+    C ABI's workspace layout: header, decode, cascade, member, append and
+    merge records, each array 256-byte aligned)."""
+    al = lambda x: (x + 255) // 256 * 256  # noqa: E731
+    off = 256
+    off = al(off + 32 * (B + 4096 + 1))
+    off = al(off + 32 * (B // 2 + 4096 + 1))
+    off = al(off + 16 * (B + 1))
+    off = al(off + 32 * (T // (64 // g) + B + 1))
+    off = al(off + 16 * (B + 1))
+    return off
+
+
+def test_long_shared_prefixes_are_measured_exactly():
+    # prompts of 562, 1025 and 1312 full pages: the prefix scan (512 page
+    # ids per step) ends in its first, second and third step; adjacent
+    # groups differ at page 0
+    rng = np.random.default_rng(77)
+    groups, gs = 3, 4
+    grp = np.repeat(np.arange(groups), gs)
+    prompt = np.array([9000, 16400, 21000])[grp]
+    S = prompt + rng.integers(1, 300, size=groups * gs)
+    b = W.build_batch("longprefix", 78, S, np.ones(len(S), np.int64), 64, 8, shared_prefix_pages=prompt // 16,
+                      prompt_lens=prompt, group_of_row=grp)
+    run, _ = _full_check(b, what="long prefixes")
+    assert run.header()["n_cascade"] > 0
+    B = b.num_seqs
+    off = _ws_lcp_offset(B, b.total_q, b.num_q_heads // b.num_kv_heads)
+    lcp = run.ws[off:off + 4 * B].view(torch.int32).cpu().numpy()
+    want = np.array([0] + [int(prompt[r]) // 16 if grp[r] == grp[r - 1] else 0 for r in range(1, B)])
+    assert np.array_equal(lcp, want), (lcp, want)
+
+
 def test_rows_without_queries_and_single_key_rows():
     b = W.build_batch("edge", 91, [1, 5, 16, 17, 40], [1, 0, 16, 0, 3], 16, 2)
     run, _ = _full_check(b, what="edge")
