@@ -869,7 +869,8 @@ def run_reference(args, rank, world):
     batch = make_batch(args.workload, "cuda" if torch.cuda.is_available() else "cpu", 0)
     stats0 = layer_stats(batch, 0, args.kv)
     nl = len(batch.layers)
-    per_step = max(2.0, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
+    # each step a bounded oracle sample; the whole run near 150 s of oracle time
+    per_step = max(0.5, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
     for w in range(args.warmup):
         cpu_baseline_sample(batch, stats0, per_step / 4, seed=1000 + w, kv=args.kv)
     vals, ms = [], []
