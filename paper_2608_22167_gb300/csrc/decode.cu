@@ -5,7 +5,7 @@
 // subgroup (NT = 4: up to 32 query vectors = members x g heads, all reading
 // the same shared prompt pages once). Per page the warp
 //   - receives the 2 KiB K block and 2 KiB V block of (page, kv head) from a
-//     per-warp ring of NSTAGE stages filled by 2-D TMA loads (128-byte
+//     per-warp ring of kDecodeStages stages filled by 2-D TMA loads (128-byte
 //     swizzle, so ldmatrix reads are bank-conflict free);
 //   - computes S^T = K Q^T with mma.sync m16n8k16 (16 keys as M, query
 //     vectors as N), masks keys outside [first_key, seq_len) on a row's
