@@ -25,6 +25,7 @@ size_t append_smem_bytes() {
 __global__ void __launch_bounds__(kAppWarps * 32)
     append_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                   const AttnParams p) {
+  if (header(p)->n_append == 0) return;  // no append rows this call
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_item;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;

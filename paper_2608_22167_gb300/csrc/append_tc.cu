@@ -170,6 +170,8 @@ __device__ __forceinline__ float chunk_probs(const uint32_t (&sv)[2][32], float 
 __global__ void __maxnreg__(144)
     append_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap qmap, const AttnParams p) {
+  // nothing to do (no append rows this call): leave before TMEM and barriers
+  if (header(p)->n_append == 0) return;
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t raw = smem_addr(smem_raw);

@@ -36,6 +36,7 @@ template <int NT>
 __global__ void __launch_bounds__(kDecodeWarps * 32)
     decode_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                   const AttnParams p) {
+  if ((NT == 1 ? header(p)->n_decode : header(p)->n_cascade) == 0) return;  // nothing of this kind
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t raw = smem_addr(smem_raw);

@@ -97,6 +97,7 @@ __device__ __forceinline__ uint32_t key_byte_mask(int c, int lo, int hi) {
 template <int NT>
 __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1)
     decode_fp8_kernel(const uint8_t* __restrict__ kv8, const AttnParams p) {
+  if ((NT == 1 ? header(p)->n_decode : header(p)->n_cascade) == 0) return;  // nothing of this kind
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
