@@ -22,16 +22,16 @@
 //              only after both PVs, so K runs a block ahead of V and the
 //              K/V loads are in flight for most of a ring's length (they
 //              often wait on HBM, which takes microseconds under load);
-//   warp 9     S issuer: S_A(b), S_B(b) = Q K_b^T (M 128, N 128, K 64, both
-//              operands K-major from shared memory);
-//   warp 10    PV issuer: O_A += P_A(b) V_b, O_B += P_B(b) V_b (M 128, N 64,
-//              K 128; P from TMEM, V MN-major from shared memory).
+//   warps 9, 10  MMA issuers of tile A and tile B: S_X(b) = Q_X K_b^T (M 128,
+//              N 128, K 64, both operands K-major from shared memory), then
+//              O_X += P_X(b - 1) V_(b-1) (M 128, N 64, K 128; P from TMEM,
+//              V MN-major from shared memory).
 // TMEM (512 columns): S_A, S_B (128 each), O_A, O_B, P_A, P_B (64 each).
 //
 // Ordering (all mbarriers, all waits bounded; X = tile A or B, phase = the
 // CTA's running block count, so no waiter can fall two phases behind):
-//   k_full/k_empty     K ring; a stage is released by the commit after S_B
-//   v_full/v_empty     V ring; a stage is released by the commit after PV_B
+//   k_full/k_empty     K ring; a stage is released by the commits after S_A, S_B
+//   v_full/v_empty     V ring; a stage is released by the commits after PV_A, PV_B
 //   s_full[X]          S_X(b) complete (commit after its 4 MMAs)
 //   s_free[X]          S_X(b) loaded into registers (4 warps arrive)
 //   p_full[X]          P_X(b) stored and O_X rescaled (4 warps arrive)
@@ -188,14 +188,14 @@ __global__ void __maxnreg__(144)
 
   if (threadIdx.x == 0) {
     mbar_init(bar(st.q_full), 1);
-    mbar_init(bar(st.q_empty), 1);
+    mbar_init(bar(st.q_empty), 2);  // one commit per tile issuer
     for (int s = 0; s < kTcKStages; ++s) {
       mbar_init(bar(st.k_full[s]), 1);
-      mbar_init(bar(st.k_empty[s]), 1);
+      mbar_init(bar(st.k_empty[s]), 2);
     }
     for (int s = 0; s < kTcVStages; ++s) {
       mbar_init(bar(st.v_full[s]), 1);
-      mbar_init(bar(st.v_empty[s]), 1);
+      mbar_init(bar(st.v_empty[s]), 2);
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(bar(st.s_full[x]), 1);
@@ -321,21 +321,26 @@ __global__ void __maxnreg__(144)
     }
   } else if (warp == kTcSWarp || warp == kTcPvWarp) {
     // ---------------------------------------------------------- MMA issuers
-    // Two issuing threads, so that neither stream waits behind the other:
-    // warp 9 issues S = Q K^T as soon as a K block and the tile's S buffer
-    // are free, warp 10 issues O += P V as each tile's P is ready. Their
-    // MMAs touch disjoint TMEM (S vs O, P) and are ordered only through the
-    // mbarriers. Both loops are lean: descriptors are computed once and
-    // stepped by constants (the start-address field counts 16-byte units and
-    // cannot overflow: shared memory ends below 256 KiB).
+    // One issuing thread per tile (warp 9: tile A, warp 10: tile B), each in
+    // its tile's own order S(b), PV(b - 1), so that neither tile's MMAs wait
+    // behind the other tile's softmax. Their MMAs touch disjoint TMEM and are
+    // ordered only through the mbarriers; a K or V stage and the query tiles
+    // are released by two commits, one per tile. The loops are lean:
+    // descriptors are computed once and stepped by constants (the
+    // start-address field counts 16-byte units and cannot overflow: shared
+    // memory ends below 256 KiB).
     if (lane == 0) {
       constexpr uint32_t idS = idesc_bf16(kTcRows, kTcKeys, false, false);
       constexpr uint32_t idO = idesc_bf16(kTcRows, kHeadDim, false, true);
       constexpr uint64_t kStageStep = kTcKvBytes / 16, kVStep = 16 * kRowBytes / 16;
-      const uint64_t qdesc[2] = {smem_desc_sw128(sQ, 16, 1024), smem_desc_sw128(sQ + kTcTileQBytes, 16, 1024)};
       const uint64_t kdesc0 = smem_desc_sw128(sK, 16, 1024);
       const uint64_t vdesc0 = smem_desc_sw128(sV, 1024, 1024);
-      const bool s_role = warp == kTcSWarp;
+      // issuer x drives tile x: S_x(b) as soon as K(b) and its S buffer are
+      // free, then O_x += P_x(b - 1) V(b - 1) once that P is ready; the two
+      // tiles never wait on each other's softmax
+      const int x = warp == kTcSWarp ? 0 : 1;
+      const uint32_t scol = tmem + col_s(x), pcol = tmem + col_p(x), ocol = tmem + col_o(x);
+      const uint64_t qd = smem_desc_sw128(sQ + x * kTcTileQBytes, 16, 1024);
       uint32_t blk = 0;
       bool ok = true;
       for (int i = 0; ok; ++i) {
@@ -346,67 +351,53 @@ __global__ void __maxnreg__(144)
         if (idx >= n_items) break;
         const int kb0 = (a.key_begin / kPage) * kPage;
         const int nb = (a.key_end - kb0 + kTcKeys - 1) / kTcKeys;
-        if (s_role) {
-          if (!wait_bar(bar(st.q_full), i & 1, abort_flag)) break;
-          for (int b = 0; b < nb; ++b, ++blk) {
-            const int s = blk % kTcKStages;
-            if (!wait_bar(bar(st.k_full[s]), (blk / kTcKStages) & 1, abort_flag)) {
+        if (!wait_bar(bar(st.q_full), i & 1, abort_flag)) break;
+        for (int b = 0; b <= nb && ok; ++b) {
+          if (b < nb) {  // S_x(b)
+            const uint32_t bk = blk + b;
+            const int s = bk % kTcKStages;
+            // S buffer x was last loaded by the softmax of block bk - 1
+            if (!wait_bar(bar(st.k_full[s]), (bk / kTcKStages) & 1, abort_flag) ||
+                (bk >= 1 && !wait_bar(bar(st.s_free[x]), (bk - 1) & 1, abort_flag))) {
               ok = false;
               break;
             }
+            tc_fence_after();
             const uint64_t kd = kdesc0 + s * kStageStep;
+            tc_mma_ss(scol, qd, kd, idS, 0u);
 #pragma unroll
-            for (int x = 0; x < 2; ++x) {
-              // S buffer X was last loaded by the softmax of block blk - 1
-              if (blk >= 1 && !wait_bar(bar(st.s_free[x]), (blk - 1) & 1, abort_flag)) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              const uint32_t scol = tmem + col_s(x);
-              tc_mma_ss(scol, qdesc[x], kd, idS, 0u);
-#pragma unroll
-              for (int kk = 1; kk < kHeadDim / 16; ++kk)
-                tc_mma_ss(scol, qdesc[x] + (uint64_t)(kk * 2), kd + (uint64_t)(kk * 2), idS, 1u);
-              tc_commit(bar(st.s_full[x]));
-            }
-            if (!ok) break;
-            tc_commit(bar(st.k_empty[s]));
-            if (b == nb - 1) tc_commit(bar(st.q_empty));
+            for (int kk = 1; kk < kHeadDim / 16; ++kk)
+              tc_mma_ss(scol, qd + (uint64_t)(kk * 2), kd + (uint64_t)(kk * 2), idS, 1u);
+            tc_commit(bar(st.s_full[x]));
+            tc_commit(bar(st.k_empty[s]));              // released when both tiles have read it
+            if (b == nb - 1) tc_commit(bar(st.q_empty));  // likewise
           }
-        } else {
-          for (int b = 0; b < nb; ++b, ++blk) {
-            const int sv = blk % kTcVStages;
-            if (!wait_bar(bar(st.v_full[sv]), (blk / kTcVStages) & 1, abort_flag)) {
+          if (b >= 1) {  // O_x += P_x(b - 1) V(b - 1)
+            const uint32_t bv = blk + b - 1;
+            const int sv = bv % kTcVStages;
+            if (!wait_bar(bar(st.v_full[sv]), (bv / kTcVStages) & 1, abort_flag) ||
+                !wait_bar(bar(st.p_full[x]), bv & 1, abort_flag) ||
+                (b == 1 && i >= 1 && !wait_bar(bar(st.o_free[x]), (i - 1) & 1, abort_flag))) {
               ok = false;
               break;
             }
+            tc_fence_after();
             const uint64_t vd = vdesc0 + sv * kStageStep;
+            tc_mma_ts(ocol, pcol, vd, idO, b > 1 ? 1u : 0u);
 #pragma unroll
-            for (int x = 0; x < 2; ++x) {
-              if (!wait_bar(bar(st.p_full[x]), blk & 1, abort_flag) ||
-                  (b == 0 && i >= 1 && !wait_bar(bar(st.o_free[x]), (i - 1) & 1, abort_flag))) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              const uint32_t pcol = tmem + col_p(x), ocol = tmem + col_o(x);
-              tc_mma_ts(ocol, pcol, vd, idO, b > 0 ? 1u : 0u);
-#pragma unroll
-              for (int kk = 1; kk < kTcKeys / 16; ++kk) tc_mma_ts(ocol, pcol + kk * 8, vd + kk * kVStep, idO, 1u);
-              tc_commit(bar(st.o_ready[x]));
-            }
-            if (!ok) break;
-            tc_commit(bar(st.v_empty[sv]));
+            for (int kk = 1; kk < kTcKeys / 16; ++kk) tc_mma_ts(ocol, pcol + kk * 8, vd + kk * kVStep, idO, 1u);
+            tc_commit(bar(st.o_ready[x]));
+            tc_commit(bar(st.v_empty[sv]));  // released when both tiles have read it
           }
         }
         if (!ok) break;
+        blk += nb;
         mbar_arrive(bar(st.item_empty[slot]));
       }
       // wait for this thread's MMAs still in flight (only after an abort can
       // any be), so that TMEM is not freed under them
-      tc_commit(bar(st.drain[s_role ? 0 : 1]));
-      mbar_wait(bar(st.drain[s_role ? 0 : 1]), 0);
+      tc_commit(bar(st.drain[x]));
+      mbar_wait(bar(st.drain[x]), 0);
     }
   } else {
     // ------------------------------------------------------------- softmax
