@@ -17,8 +17,9 @@
  *
  * Conventions shared by every entry point
  * ---------------------------------------
- *  - Every pointer argument except `dims`/`opts`/`status_bits` is DEVICE
- *    memory owned by the caller; the library never frees or retains it.
+ *  - Every pointer argument except `dims`/`opts`/`status_bits` and the
+ *    `*_host` arguments of mcpu_paged_attention_host is DEVICE memory owned
+ *    by the caller; the library never frees or retains it.
  *    Tensors are dense, row-major, with the shapes given below. bf16 data and
  *    the pools must be 16-byte aligned.
  *  - Work is enqueued on `stream` (NULL = the legacy default stream) and the
@@ -246,13 +247,20 @@ mcpu_status mcpu_grow_block_tables(int32_t* block_table, const int32_t* seq_lens
  *
  * Layout: one pool `kv8` of num_pages * H_kv blocks of 2176 bytes, block
  * (page, h) at byte offset (page * H_kv + h) * 2176 (16-byte aligned base):
- *   bytes    0..1023  K codes, uint8 [16 slots][D]
- *   bytes 1024..2047  V codes, uint8 [D][16 slots]   (transposed)
- *   bytes 2048..2111  K scales, float [16 slots]
- *   bytes 2112..2175  V scales, float [16 slots]
+ *   bytes    0..1023  K codes, uint8 [16 slots][D] (row-major)
+ *   bytes 1024..2047  V codes in the decode kernel's MMA-fragment order: for
+ *                     half e in {0, 1}, lane l = 4 r + c (r in 0..7, c in
+ *                     0..3), j in 0..3 and i in 0..3, byte
+ *                     1024 + 512 e + 16 l + 4 j + i holds dim
+ *                     16 (2 e + j / 2) + 8 (j % 2) + r of slot 4 c + i
+ *   bytes 2048..2175  scales, float: for r in 0..7, the 16 bytes at
+ *                     2048 + 16 r hold the K scales of slots a and a + 2,
+ *                     then the V scales of slots a and a + 2, where
+ *                     a = 4 (r / 2) + r % 2
  * so that one copy brings a page's K, V and scales (a 16-token page takes
- * 2176 bytes per kv head instead of 4096 in bf16). Slots that no row has
- * written may hold anything: the kernels mask them.
+ * 2176 bytes per kv head instead of 4096 in bf16) and every operand of a
+ * lane is one 16-byte shared-memory load. Slots that no row has written may
+ * hold anything: the kernels mask them.
  *
  * mcpu_kv_append_fp8: as mcpu_kv_append (same placement, lengths and error
  * bits), quantizing each new K and V row as above; k_new, v_new stay bf16.
@@ -266,10 +274,11 @@ mcpu_status mcpu_kv_append_fp8(const void* k_new, const void* v_new, void* kv8, 
  * 0): same arguments, results and options as mcpu_paged_attention_forward
  * (split-KV, cascade pass over shared prompt pages, sliding window, sinks,
  * phase events, graph capture), with the two bf16 pools replaced by kv8.
- * dims->num_pages counts pages of kv8. The products run on the fp8 tensor
- * cores: q is carried as three e4m3 pieces (exact to about 2^-12 of a query
- * vector's largest entry) and the softmax weights times the V scales as two
- * (fp16 rounded, then to about 2^-8 relative), accumulation in fp32.
+ * dims->num_pages counts pages of kv8. The products run on the fp16 tensor
+ * cores: codes are converted exactly to fp16; q enters as fp16 times a power
+ * of two per query vector (exact for every bf16 entry above 2^-28 of the
+ * vector's largest); the softmax weights times the V scales enter as fp16
+ * (about 2^-11 relative); accumulation in fp32.
  * A batch with total_q > num_seqs (some row appends) returns
  * MCPU_ERR_UNSUPPORTED without launching; an append row found on the device
  * is skipped and reported as MCPU_ERR_UNSUPPORTED_ROW. MCPU_FLAG_MMA_SYNC_APPEND
@@ -280,6 +289,75 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
                                              int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
                                              void* out, float* lse, void* workspace, size_t workspace_bytes,
                                              const mcpu_options* opts, mcpu_stream_t stream);
+
+/*
+ * Calls with host buffers (a deployment variant with no counterpart in the
+ * paper, whose engine keeps q, K and V on the GPU): one layer's per-token
+ * inputs and outputs live in host memory and the library moves them, with
+ * the copies overlapped with the attention itself.
+ *
+ * mcpu_host_stage_create allocates, on the current device, `slots` (2 to
+ * MCPU_MAX_HOST_SLOTS) staging slots of device memory (each holds one
+ * call's q, k_new, v_new, out, lse and row metadata for up to max_tokens
+ * query tokens and max_rows rows with the given head counts; about
+ * max_tokens * (4 H_q + 2 H_kv) * 64 bytes each) and two copy streams.
+ * Calls take the slots in turn, so the inputs of the next slots - 1 calls
+ * can be copied in while one computes (more slots absorb layers whose
+ * copies outlast their compute). Returns MCPU_ERR_CUDA if an allocation
+ * fails. mcpu_host_stage_destroy waits for
+ * the stage's copies and frees it (NULL is ignored).
+ *
+ * mcpu_paged_attention_host: mcpu_kv_append followed by
+ * mcpu_paged_attention_forward (same arguments, rules and results) with
+ *   q_host [T, H_q, D], k_new_host / v_new_host [T, H_kv, D] bf16,
+ *   seq_lens_host [B], query_start_loc_host [B + 1] int32: HOST memory;
+ *   out_host [T, H_q, D] bf16, lse_host [T, H_q] float: HOST memory;
+ *   k_cache, v_cache, block_table, workspace: device memory as before.
+ * The rows are cut into `slices` contiguous row ranges of about equal token
+ * counts (mcpu_host_slice_rows; at most MCPU_MAX_HOST_SLICES; 0 = two
+ * slices from 64 MiB moved, else one; a single row is never cut). Slice s's inputs are copied in on the
+ * stage's input stream while slice s - 1 computes, and its outputs are
+ * copied out on the output stream while slice s + 1 computes; the compute
+ * runs on `stream`, ordered after the work already there. Shared-prefix
+ * detection only sees rows within one slice. query_start_loc_host is read
+ * on the host during the call; the other host buffers are read or written
+ * asynchronously: page-locked memory gives full copy speed, and every host
+ * buffer must stay valid, and the inputs unchanged, until the outputs are
+ * complete. The outputs of a call are complete once mcpu_host_stage_sync
+ * has returned, or, on the device, after a later mcpu_host_stage_wait on
+ * `stream`. A stage serves one calling thread at a time. Errors: the
+ * checks of the two wrapped calls, plus
+ * MCPU_ERR_INVALID_ARG when the call exceeds the stage's capacity or head
+ * counts, or the current device is not the stage's.
+ */
+#define MCPU_MAX_HOST_SLICES 8
+#define MCPU_MAX_HOST_SLOTS 4
+typedef struct mcpu_host_stage mcpu_host_stage;
+mcpu_status mcpu_host_stage_create(int32_t max_tokens, int32_t max_rows, int32_t num_q_heads, int32_t num_kv_heads,
+                                   int32_t slots, mcpu_host_stage** stage);
+mcpu_status mcpu_host_stage_destroy(mcpu_host_stage* stage);
+mcpu_status mcpu_paged_attention_host(mcpu_host_stage* stage, const void* q_host, const void* k_new_host,
+                                      const void* v_new_host, void* k_cache, void* v_cache,
+                                      const int32_t* block_table, const int32_t* seq_lens_host,
+                                      const int32_t* query_start_loc_host, int32_t sliding_window,
+                                      float softmax_scale, const mcpu_dims* dims, void* out_host, float* lse_host,
+                                      void* workspace, size_t workspace_bytes, const mcpu_options* opts,
+                                      int32_t slices, mcpu_stream_t stream);
+/* The row ranges mcpu_paged_attention_host uses for `slices` > 0 slices:
+ * writes row_begin[0 .. n] (row_begin[0] = 0, row_begin[n] = num_seqs,
+ * strictly increasing) and returns the number n of non-empty slices (0 for
+ * no rows or invalid arguments). Boundary k is the row whose first token is
+ * nearest to k / slices of the total (query_start_loc_host [B + 1], host
+ * memory), after the previous boundary; a slice without tokens is dropped.
+ * row_begin needs room for slices + 1 entries. Host only. */
+int32_t mcpu_host_slice_rows(const int32_t* query_start_loc_host, int32_t num_seqs, int32_t slices,
+                             int32_t* row_begin);
+/* Makes `stream` wait (on the device) for every output copy the stage has
+ * enqueued so far. */
+mcpu_status mcpu_host_stage_wait(mcpu_host_stage* stage, mcpu_stream_t stream);
+/* Blocks the calling thread until every output copy the stage has enqueued
+ * so far is complete. */
+mcpu_status mcpu_host_stage_sync(mcpu_host_stage* stage);
 
 /* Synchronises `stream`, reads the workspace status word and maps it to the
  * most severe mcpu_status (MCPU_OK if clear). The raw bits go to
@@ -298,7 +376,7 @@ const char* mcpu_status_string(mcpu_status status);
  * failed. Not cleared by later successful calls. */
 int32_t mcpu_last_cuda_error(void);
 
-/* Version of this ABI (bumped on any signature change). */
+/* Version of this ABI (bumped on any signature change or addition). */
 int32_t mcpu_abi_version(void);
 
 #ifdef __cplusplus

@@ -115,6 +115,25 @@ _lib.mcpu_abi_version.argtypes = []
 _lib.mcpu_abi_version.restype = ctypes.c_int32
 _lib.mcpu_last_cuda_error.argtypes = []
 _lib.mcpu_last_cuda_error.restype = ctypes.c_int32
+_lib.mcpu_host_stage_create.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                        ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]
+_lib.mcpu_host_stage_create.restype = ctypes.c_int
+_lib.mcpu_host_stage_destroy.argtypes = [_P]
+_lib.mcpu_host_stage_destroy.restype = ctypes.c_int
+_lib.mcpu_host_stage_wait.argtypes = [_P, _P]
+_lib.mcpu_host_stage_wait.restype = ctypes.c_int
+_lib.mcpu_host_stage_sync.argtypes = [_P]
+_lib.mcpu_host_stage_sync.restype = ctypes.c_int
+_lib.mcpu_host_slice_rows.argtypes = [_P, ctypes.c_int32, ctypes.c_int32, _P]
+_lib.mcpu_host_slice_rows.restype = ctypes.c_int32
+_lib.mcpu_paged_attention_host.argtypes = [
+    _P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P,
+    ctypes.c_size_t, ctypes.POINTER(Options), ctypes.c_int32, _P,
+]
+_lib.mcpu_paged_attention_host.restype = ctypes.c_int
+
+MAX_HOST_SLICES = 8
+MAX_HOST_SLOTS = 4
 
 
 def _ptr(t):
@@ -328,3 +347,87 @@ def new_workspace(d: Dims, device="cuda") -> torch.Tensor:
 def status_word(workspace) -> torch.Tensor:
     """The device int32 status word at the start of a workspace."""
     return workspace[:4].view(torch.int32)
+
+
+# ---------------------------------------------------------------- host buffers
+class HostStage:
+    """Handle of an mcpu_host_stage: device staging for calls with host
+    buffers (see mcpu_paged_attention_host). Keeps the host tensors of every
+    call made since the last sync() alive."""
+
+    def __init__(self, max_tokens, max_rows, num_q_heads, num_kv_heads, slots=2):
+        h = ctypes.c_void_p()
+        _check(_lib.mcpu_host_stage_create(int(max_tokens), int(max_rows), int(num_q_heads), int(num_kv_heads),
+                                           int(slots), ctypes.byref(h)), "mcpu_host_stage_create")
+        self.handle = h
+        self._pending = []
+
+    def close(self):
+        if self.handle:
+            _lib.mcpu_host_stage_destroy(self.handle)
+            self.handle = None
+            self._pending = []
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def mcpu_host_stage_create(max_tokens, max_rows, num_q_heads, num_kv_heads, slots=2) -> HostStage:
+    return HostStage(max_tokens, max_rows, num_q_heads, num_kv_heads, slots)
+
+
+def mcpu_host_stage_destroy(stage: HostStage):
+    stage.close()
+
+
+def mcpu_host_stage_wait(stage: HostStage, stream=None):
+    _check(_lib.mcpu_host_stage_wait(stage.handle, _stream(stream)), "mcpu_host_stage_wait")
+
+
+def mcpu_host_stage_sync(stage: HostStage):
+    _check(_lib.mcpu_host_stage_sync(stage.handle), "mcpu_host_stage_sync")
+    stage._pending = []
+
+
+def _host_i32(t):
+    if t.is_cuda or t.dtype != torch.int32 or not t.is_contiguous():
+        raise ValueError("expected a contiguous int32 host tensor")
+    return t
+
+
+def mcpu_host_slice_rows(query_start_loc_host, slices):
+    """Row boundaries [0, ..., B] of the slices mcpu_paged_attention_host uses."""
+    qsl = _host_i32(query_start_loc_host)
+    rb = (ctypes.c_int32 * (MAX_HOST_SLICES + 1))()
+    n = int(_lib.mcpu_host_slice_rows(_ptr(qsl), int(qsl.numel()) - 1, int(slices), ctypes.cast(rb, _P)))
+    return [int(rb[i]) for i in range(n + 1)] if n > 0 else []
+
+
+def mcpu_paged_attention_host(stage, q_host, k_new_host, v_new_host, k_cache, v_cache, block_table, seq_lens_host,
+                              query_start_loc_host, sliding_window, softmax_scale, out_host, lse_host, workspace,
+                              flags=0, split_pages=0, slices=0, stream=None, sinks=None):
+    """KV append and forward of one layer whose q / k_new / v_new and out /
+    lse are host (CPU) tensors, page-locked for full copy speed; seq_lens
+    and query_start_loc are int32 host tensors; pools, block table and
+    workspace stay on the device. The outputs are complete after
+    mcpu_host_stage_sync(stage) (or, on the device, after
+    mcpu_host_stage_wait(stage, stream))."""
+    for t in (q_host, k_new_host, v_new_host, out_host, lse_host):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError("q / k_new / v_new / out / lse must be contiguous host tensors")
+    sl, qsl = _host_i32(seq_lens_host), _host_i32(query_start_loc_host)
+    d = dims(q_host, k_cache, block_table, sl)
+    opts = _options(d.num_q_heads, flags, split_pages, None, sinks)
+    _check(
+        _lib.mcpu_paged_attention_host(
+            stage.handle, _ptr(q_host), _ptr(k_new_host), _ptr(v_new_host), _ptr(k_cache), _ptr(v_cache),
+            _ptr(block_table), _ptr(sl), _ptr(qsl), int(sliding_window), float(softmax_scale), ctypes.byref(d),
+            _ptr(out_host), _ptr(lse_host), _ptr(workspace), int(workspace.numel() * workspace.element_size()),
+            ctypes.byref(opts), int(slices), _stream(stream),
+        ),
+        "mcpu_paged_attention_host",
+    )
+    stage._pending.append((q_host, k_new_host, v_new_host, out_host, lse_host, sl, qsl, opts))

@@ -162,3 +162,71 @@ def test_no_gpu_is_a_clean_error(lib):
     need = lib.mcpu_workspace_size(ctypes.byref(d))
     P = 1 << 20
     assert fwd(P, P, P, P, P, P, 0, 0.125, ctypes.byref(d), P, P, P, need, None, None) == 4
+
+
+def test_host_slice_rows(lib):
+    # row ranges of the host-buffer call: 0 .. B, strictly increasing, every
+    # slice with tokens, each boundary the row start nearest its target
+    import numpy as np
+
+    f = lib.mcpu_host_slice_rows
+    f.restype = ctypes.c_int32
+    rng = np.random.default_rng(11)
+    for trial in range(300):
+        B = int(rng.integers(1, 40))
+        L = rng.integers(0, 50, size=B)
+        L[rng.random(B) < 0.2] = int(rng.integers(100, 2000))
+        qsl = np.concatenate([[0], np.cumsum(L)]).astype(np.int32)
+        T = int(qsl[-1])
+        for slices in range(1, 9):
+            rb = (ctypes.c_int32 * 9)()
+            n = f(qsl.ctypes.data_as(ctypes.c_void_p), B, slices, ctypes.cast(rb, ctypes.c_void_p))
+            got = [rb[i] for i in range(n + 1)]
+            if T == 0:
+                assert n == 1 and got == [0, B]
+                continue
+            assert 1 <= n <= slices and got[0] == 0 and got[-1] == B
+            assert all(a < b for a, b in zip(got, got[1:]))
+            for a, b in zip(got[:-2], got[1:-1]):  # interior slices carry tokens
+                assert qsl[b] > qsl[a]
+            # brute force: boundary k is the row start nearest round(T k / slices) after the last one
+            exp = [0]
+            for k in range(1, slices):
+                target = (T * k + slices // 2) // slices
+                cands = range(exp[-1] + 1, B)
+                if not cands:
+                    continue
+                lo = next((r for r in cands if qsl[r] >= target), B)
+                if lo - 1 > exp[-1] and target - qsl[lo - 1] < qsl[lo] - target:
+                    lo -= 1
+                if lo < B and qsl[lo] > qsl[exp[-1]]:
+                    exp.append(lo)
+            exp.append(B)
+            assert got == exp, (qsl.tolist(), slices, got, exp)
+    rb = (ctypes.c_int32 * 9)()
+    qsl = np.zeros(1, np.int32)
+    assert f(qsl.ctypes.data_as(ctypes.c_void_p), 0, 4, ctypes.cast(rb, ctypes.c_void_p)) == 0
+    assert f(qsl.ctypes.data_as(ctypes.c_void_p), 0, 9, ctypes.cast(rb, ctypes.c_void_p)) == 0
+    assert f(None, 3, 2, ctypes.cast(rb, ctypes.c_void_p)) == 0
+
+
+def test_host_stage_host_checks(lib):
+    # checks that return before any CUDA call: no stage, bad sizes
+    null = ctypes.c_void_p()
+    assert _fn(lib, "mcpu_host_stage_wait")(null, null) == 1
+    assert _fn(lib, "mcpu_host_stage_sync")(null) == 1
+    assert _fn(lib, "mcpu_host_stage_destroy")(null) == 0
+    h = ctypes.c_void_p()
+    create = _fn(lib, "mcpu_host_stage_create")
+    assert create(0, 4, 8, 2, 2, ctypes.byref(h)) == 1
+    assert create(16, 4, 8, 3, 2, ctypes.byref(h)) == 1  # H_q not a multiple of H_kv
+    assert create(16, 4, 8, 2, 1, ctypes.byref(h)) == 1  # fewer than two slots
+    assert create(16, 4, 8, 2, 5, ctypes.byref(h)) == 1  # more than MCPU_MAX_HOST_SLOTS
+    assert create(16, 4, 8, 2, 2, None) == 1
+    d = Dims(4, 4, 19, 34, 8, 2, 64, 16)
+    call = _fn(lib, "mcpu_paged_attention_host")
+    call.argtypes = [ctypes.c_void_p] * 9 + [ctypes.c_int32, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
+                                             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p,
+                                             ctypes.c_int32, ctypes.c_void_p]
+    assert call(None, None, None, None, None, None, None, None, None, 0, 0.125, ctypes.byref(d), None, None, None,
+                0, None, 0, None) == 1
