@@ -325,7 +325,10 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
  * buffer must stay valid, and the inputs unchanged, until the outputs are
  * complete. The outputs of a call are complete once mcpu_host_stage_sync
  * has returned, or, on the device, after a later mcpu_host_stage_wait on
- * `stream`. A stage serves one calling thread at a time. Errors: the
+ * `stream`. A stage serves one calling thread at a time. An error after the
+ * call has begun enqueuing leaves the stage usable (its later calls and
+ * mcpu_host_stage_sync wait for what was enqueued); the outputs are then
+ * undefined. mcpu_host_stage_destroy waits for every call's work. Errors: the
  * checks of the two wrapped calls, plus
  * MCPU_ERR_INVALID_ARG when the call exceeds the stage's capacity or head
  * counts, or the current device is not the stage's.

@@ -51,6 +51,8 @@ struct mcpu_host_stage {
 namespace {
 
 void release(mcpu_host_stage* hs) {
+  // the output stream's last event follows every call's compute and copies
+  if (hs->any_out) cudaEventSynchronize(hs->ev_out);
   if (hs->in) cudaStreamSynchronize(hs->in);
   if (hs->out) cudaStreamSynchronize(hs->out);
   for (Slot& s : hs->slot) {
@@ -72,6 +74,21 @@ void release(mcpu_host_stage* hs) {
 bool on_stage_device(const mcpu_host_stage* hs) {
   int dev = -1;
   return cudaGetDevice(&dev) == cudaSuccess && dev == hs->device;
+}
+
+// After a failure part-way through a call: the slot is released, and the
+// stage's output event placed, only after everything the call enqueued on
+// the input, compute and output streams (best effort, errors ignored), so
+// that no later call overwrites staging that is still in use.
+mcpu_status fail_after_enqueue(mcpu_host_stage* hs, Slot& sl, cudaStream_t s, mcpu_status st) {
+  cudaEventRecord(hs->ev_in[0], hs->in);
+  cudaStreamWaitEvent(hs->out, hs->ev_in[0], 0);
+  cudaEventRecord(hs->ev_done[0], s);
+  cudaStreamWaitEvent(hs->out, hs->ev_done[0], 0);
+  cudaEventRecord(sl.free, hs->out);
+  cudaEventRecord(hs->ev_out, hs->out);
+  hs->any_out = true;
+  return st;
 }
 
 }  // namespace
@@ -222,8 +239,8 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(sl.qsl, sl.qsl_host, (size_t)(B + n) * 4, cudaMemcpyHostToDevice, hs->in);
   if (e == cudaSuccess) e = cudaEventRecord(sl.meta_copied, hs->in);
-  if (e != cudaSuccess) return MCPU_ERR_CUDA;
   sl.used = true;
+  if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
 
   const uint8_t* qh = static_cast<const uint8_t*>(q_host);
   const uint8_t* knh = static_cast<const uint8_t*>(k_new_host);
@@ -241,7 +258,7 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
       e = cudaMemcpyAsync(sl.vn + t0 * kv_row, vnh + t0 * kv_row, nt * kv_row, cudaMemcpyHostToDevice, hs->in);
     if (e == cudaSuccess) e = cudaEventRecord(hs->ev_in[k], hs->in);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(s, hs->ev_in[k], 0);
-    if (e != cudaSuccess) return MCPU_ERR_CUDA;
+    if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
     // the slice's KV append and forward on the caller's stream
     mcpu_dims d = *dims;
     d.num_seqs = b - a;
@@ -250,12 +267,12 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
     const int32_t* qsl = sl.qsl + a + k;
     mcpu_status st = mcpu_kv_append(sl.kn + t0 * kv_row, sl.vn + t0 * kv_row, k_cache, v_cache, bt, sl.sl + a, qsl,
                                     &d, static_cast<int32_t*>(workspace), stream);
-    if (st != MCPU_OK) return st;
+    if (st != MCPU_OK) return fail_after_enqueue(hs, sl, s, st);
     st = mcpu_paged_attention_forward(sl.q + t0 * q_row, k_cache, v_cache, bt, sl.sl + a, qsl, sliding_window,
                                       softmax_scale, &d, sl.out + t0 * q_row,
                                       reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sl.lse) + t0 * lse_row),
                                       workspace, workspace_bytes, opts, stream);
-    if (st != MCPU_OK) return st;
+    if (st != MCPU_OK) return fail_after_enqueue(hs, sl, s, st);
     // its outputs, once computed
     e = cudaEventRecord(hs->ev_done[k], s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(hs->out, hs->ev_done[k], 0);
@@ -264,11 +281,11 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
     if (e == cudaSuccess)
       e = cudaMemcpyAsync(lh + t0 * lse_row, reinterpret_cast<uint8_t*>(sl.lse) + t0 * lse_row, nt * lse_row,
                           cudaMemcpyDeviceToHost, hs->out);
-    if (e != cudaSuccess) return MCPU_ERR_CUDA;
+    if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
   }
   e = cudaEventRecord(sl.free, hs->out);
   if (e == cudaSuccess) e = cudaEventRecord(hs->ev_out, hs->out);
-  if (e != cudaSuccess) return MCPU_ERR_CUDA;
+  if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
   hs->any_out = true;
   return MCPU_OK;
 }
