@@ -304,8 +304,7 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
  * Calls take the slots in turn, so the inputs of the next slots - 1 calls
  * can be copied in while one computes (more slots absorb layers whose
  * copies outlast their compute). Returns MCPU_ERR_CUDA if an allocation
- * fails. mcpu_host_stage_destroy waits for
- * the stage's copies and frees it (NULL is ignored).
+ * fails. mcpu_host_stage_destroy frees the stage (NULL is ignored).
  *
  * mcpu_paged_attention_host: mcpu_kv_append followed by
  * mcpu_paged_attention_forward (same arguments, rules and results) with
