@@ -11,7 +11,7 @@ pytestmark = pytest.mark.gpu
 
 if torch.cuda.is_available():
     import oracle
-    from _gpu import Fp8Run, assert_parity
+    from _gpu import Fp8Run, assert_parity, from_fp8_blocks, oracle_quantize_pool, to_fp8_blocks
     from paper_2608_22167_gb300 import mcpu
 
 
@@ -225,6 +225,68 @@ def test_decode_batch_sampled_at_full_size():
                                                 h["query_start_loc"], 0, h["softmax_scale"], toks, heads)
     go, gl = run.out_host()
     assert_parity(go[toks, heads], gl[toks, heads], oracle.bf16_bits_to_float(ro), rl, "decode_b64 fp8")
+
+
+def _device_quantized_pool(pool, device="cuda"):
+    """An fp8 pool holding every page of a bf16 pool, written on the device by
+    mcpu_kv_append_fp8 (each page appended as one 16-token row). Only the
+    unchecked rows' pages keep these codes."""
+    P, H, page, D = pool.k_cache.shape
+    kv8 = mcpu.new_fp8_pool(P, H, device)
+    status = torch.zeros(1, dtype=torch.int32, device=device)
+    for p0 in range(0, P, 2048):
+        n = min(2048, P - p0)
+        kn = pool.k_cache[p0:p0 + n].permute(0, 2, 1, 3).reshape(n * page, H, D).contiguous()
+        vn = pool.v_cache[p0:p0 + n].permute(0, 2, 1, 3).reshape(n * page, H, D).contiguous()
+        bt = torch.arange(p0, p0 + n, dtype=torch.int32, device=device).view(n, 1)
+        sl = torch.full((n,), page, dtype=torch.int32, device=device)
+        qsl = torch.arange(0, (n + 1) * page, page, dtype=torch.int32, device=device)
+        mcpu.mcpu_kv_append_fp8(kn, vn, kv8, bt, sl, qsl, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    return kv8
+
+
+def test_long_batch_sampled_at_full_size():
+    # the long-horizon batch (512 rows, 33 GB of bf16 KV) over fp8 pages, in
+    # the bench's launch configuration. The checked rows' pages hold the
+    # oracle's codes; the rest of the pool is quantized on the device.
+    b = W.config_long(device="cuda")
+    lay = b.layers[0]
+    pool = b.pools[lay.pool]
+    order = np.argsort(b.seq_lens)
+    rows = sorted(set(int(r) for r in list(order[:2]) + list(order[-3:]) + list(order[256:259])))
+    h = W.host_rows(b, rows)
+    bt_rows = pool.block_table[rows]
+    used = np.unique(bt_rows[bt_rows >= 0])  # compact page i of h is physical page used[i]
+    before = oracle_quantize_pool(h["k_cache"], h["v_cache"])
+    kv8 = _device_quantized_pool(pool)
+    used_t = torch.as_tensor(used.astype(np.int64), device="cuda")
+    kv8.index_copy_(0, used_t, torch.from_numpy(to_fp8_blocks(*before)).to("cuda"))
+    bt = torch.from_numpy(pool.block_table).to("cuda")
+    sl = torch.from_numpy(b.seq_lens).to("cuda")
+    qsl = torch.from_numpy(b.query_start_loc).to("cuda")
+    ws = mcpu.new_workspace(mcpu.dims_fp8(lay.q, kv8, bt, sl), "cuda")
+    out = torch.full_like(lay.q, float("nan"))
+    lse = torch.full(lay.q.shape[:2], float("nan"), dtype=torch.float32, device="cuda")
+    mcpu.mcpu_kv_append_fp8(lay.k_new, lay.v_new, kv8, bt, sl, qsl, mcpu.status_word(ws))
+    mcpu.mcpu_paged_attention_forward_fp8(lay.q, kv8, bt, sl, qsl, 0, b.softmax_scale, out, lse, ws)
+    code, bits = mcpu.mcpu_read_device_status(ws)
+    assert code == 0, f"device status bits {bits}"
+    after = oracle.kv_append_fp8(h["k_new"], h["v_new"], *before, h["block_table"], h["seq_lens"],
+                                 h["query_start_loc"])
+    got = from_fp8_blocks(kv8.index_select(0, used_t).cpu().numpy())
+    for g, r, what in zip(got, after, ("k codes", "v codes", "k scales", "v scales")):
+        assert np.array_equal(np.ascontiguousarray(g).view(np.uint8), np.ascontiguousarray(r).view(np.uint8)), what
+    n_tok = int(h["query_start_loc"][-1])
+    toks = np.repeat(np.arange(n_tok, dtype=np.int64), b.num_q_heads)
+    heads = np.tile(np.arange(b.num_q_heads, dtype=np.int32), n_tok)
+    ro, rl = oracle.paged_attention_sampled_fp8(h["q"], *after, h["block_table"], h["seq_lens"],
+                                                h["query_start_loc"], 0, h["softmax_scale"], toks, heads)
+    full = h["token_map"][toks]
+    go = out.float().cpu().numpy()[full, heads]
+    gl = lse.cpu().numpy()[full, heads]
+    assert_parity(go, gl, oracle.bf16_bits_to_float(ro), rl, "long_b512 fp8")
 
 
 def test_fp8_and_bf16_paths_agree_on_exactly_representable_pools():

@@ -66,6 +66,27 @@ def test_host_call_matches_oracle(seed, slices):
     st.close()
 
 
+@pytest.mark.parametrize("window", [0, 16, 128])
+def test_host_call_with_sinks_and_windows(window):
+    # options reach every slice: attention sinks, and a sliding window
+    rng = np.random.default_rng(3600 + window)
+    S = rng.integers(20, 1500, size=7)
+    L = np.where(rng.random(7) < 0.5, 1, np.minimum(S, rng.integers(2, 200, size=7)))
+    b = W.build_batch("host_sinks", 3600 + window, S, L, 16, 2, layer_windows=(window,))
+    sinks = rng.normal(0.0, 2.0, size=16).astype(np.float32)
+    hc = HostCall(b)
+    st = hc.stage()
+    mcpu.mcpu_paged_attention_host(st, hc.q, hc.k_new, hc.v_new, hc.kc, hc.vc, hc.bt, hc.sl, hc.qsl, hc.window,
+                                   b.softmax_scale, hc.out, hc.lse, hc.ws, slices=3,
+                                   sinks=torch.from_numpy(sinks).to("cuda"))
+    mcpu.mcpu_host_stage_sync(st)
+    code, bits = mcpu.mcpu_read_device_status(hc.ws)
+    assert code == 0, f"device status bits {bits}"
+    ref_out, ref_lse, _ = oracle_full(b, 0, sinks=sinks)
+    assert_parity(hc.out.float().numpy(), hc.lse.numpy(), ref_out, ref_lse, f"sinks window={window}")
+    st.close()
+
+
 def test_host_call_pageable_buffers():
     # page-locked memory is the fast path, ordinary host memory must work too
     b = W.fuzz_batch(3100, max_len=800, max_chunk=100)
