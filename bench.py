@@ -634,52 +634,42 @@ def run_ours(args, rank, world, dev):
     cands = [r for r in (roof_dec, roof_app) if r is not None]
     dominant = max(cands, key=lambda r: r["ms_per_step"]) if cands else None
 
-    # ---- end to end: host buffers, copies inside the timed region. bf16
-    # pools: every layer through mcpu_paged_attention_host (the library
+    # ---- end to end: host buffers, copies inside the timed region: every
+    # layer through mcpu_paged_attention_host (_fp8 over fp8 pools), which
     # copies q / k_new / v_new in and out / lse back, overlapped with the
-    # compute by row slices); the step ends when its last output is in host
-    # memory. fp8 pools: torch copies around the device calls.
+    # compute by row slices; the step ends when its last output is in host
+    # memory.
     lay_host = []
     for lay in batch.layers:
         lay_host.append((lay.q.cpu().pin_memory(), lay.k_new.cpu().pin_memory(), lay.v_new.cpu().pin_memory()))
     meta_host = [torch.from_numpy(batch.seq_lens).to(torch.int32).pin_memory(),
                  torch.from_numpy(batch.query_start_loc).to(torch.int32).pin_memory()]
     bt_host = {k: torch.from_numpy(p.block_table).pin_memory() for k, p in batch.pools.items()}
-    q_d = torch.empty_like(batch.layers[0].q)
-    kn_d = torch.empty_like(batch.layers[0].k_new)
-    vn_d = torch.empty_like(batch.layers[0].v_new)
-    out_h = torch.empty(q_d.shape, dtype=q_d.dtype).pin_memory()
-    lse_h = torch.empty(q_d.shape[:2], dtype=torch.float32).pin_memory()
+    q0 = batch.layers[0].q
+    out_h = torch.empty(q0.shape, dtype=q0.dtype).pin_memory()
+    lse_h = torch.empty(q0.shape[:2], dtype=torch.float32).pin_memory()
     h2d = sum(t.numel() * t.element_size() for tr in lay_host for t in tr)
     h2d += sum(t.numel() * t.element_size() for t in meta_host) + sum(
         t.numel() * t.element_size() for t in bt_host.values())
     d2h = (out_h.numel() * out_h.element_size() + lse_h.numel() * 4) * nl
-    host_stage = None if fp8 else mcpu.HostStage(q_d.shape[0], batch.num_seqs, batch.num_q_heads,
-                                                  batch.num_kv_heads, slots=3)
+    host_stage = mcpu.HostStage(q0.shape[0], batch.num_seqs, batch.num_q_heads, batch.num_kv_heads, slots=3)
 
     def e2e_step():
         for key, t in bt_host.items():
             st.bts[key].copy_(t, non_blocking=True)
-        if host_stage is not None:
-            for i in range(nl):
-                lay = batch.layers[i]
+        for i in range(nl):
+            lay = batch.layers[i]
+            qh, knh, vnh = lay_host[i]
+            if fp8:
+                mcpu.mcpu_paged_attention_host_fp8(host_stage, qh, knh, vnh, st.pools8[lay.pool], st.bts[lay.pool],
+                                                   meta_host[0], meta_host[1], lay.sliding_window,
+                                                   batch.softmax_scale, out_h, lse_h, st.ws)
+            else:
                 pool = batch.pools[lay.pool]
-                qh, knh, vnh = lay_host[i]
                 mcpu.mcpu_paged_attention_host(host_stage, qh, knh, vnh, pool.k_cache, pool.v_cache,
                                                st.bts[lay.pool], meta_host[0], meta_host[1], lay.sliding_window,
                                                batch.softmax_scale, out_h, lse_h, st.ws)
-            mcpu.mcpu_host_stage_wait(host_stage)
-            return
-        st.sl.copy_(meta_host[0], non_blocking=True)
-        st.qsl.copy_(meta_host[1], non_blocking=True)
-        for i in range(nl):
-            qh, knh, vnh = lay_host[i]
-            q_d.copy_(qh, non_blocking=True)
-            kn_d.copy_(knh, non_blocking=True)
-            vn_d.copy_(vnh, non_blocking=True)
-            st.layer_call(i, q=q_d, k_new=kn_d, v_new=vn_d)
-            out_h.copy_(st.out, non_blocking=True)
-            lse_h.copy_(st.lse, non_blocking=True)
+        mcpu.mcpu_host_stage_wait(host_stage)
 
     e2e_steps = max(3, min(args.steps, 20))
     for _ in range(2):
@@ -698,9 +688,8 @@ def run_ours(args, rank, world, dev):
     # working set can stall for a pass (plain copies do too); the median
     # shows a typical step, the mean (the reported value) includes stalls
     e2e_median_ms = statistics.median(ev[k].elapsed_time(ev[k + 1]) for k in range(e2e_steps))
-    if host_stage is not None:
-        mcpu.mcpu_host_stage_sync(host_stage)
-        host_stage.close()
+    mcpu.mcpu_host_stage_sync(host_stage)
+    host_stage.close()
 
     # ---- max over ranks
     total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], dev, world)
@@ -759,9 +748,8 @@ def run_ours(args, rank, world, dev):
         "e2e": {"value": round(e2e_value, 2), "unit": "GB/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_ms, 4),
                 "median_step_ms": round(e2e_median_ms, 4),
-                "call": ("torch copies around mcpu_paged_attention_forward_fp8" if fp8 else
-                         "mcpu_paged_attention_host per layer (host q/k_new/v_new/out/lse; copies overlapped "
-                         "with compute by row slices)")},
+                "call": ("mcpu_paged_attention_host_fp8" if fp8 else "mcpu_paged_attention_host") +
+                        " per layer (host q/k_new/v_new/out/lse; copies overlapped with compute by row slices)"},
         "clocks": clocks,
         "wall_s_timed": round(wall, 3),
     }

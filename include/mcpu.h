@@ -345,6 +345,15 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* stage, const void* q_host
                                       float softmax_scale, const mcpu_dims* dims, void* out_host, float* lse_host,
                                       void* workspace, size_t workspace_bytes, const mcpu_options* opts,
                                       int32_t slices, mcpu_stream_t stream);
+/* mcpu_paged_attention_host over fp8 pages: mcpu_kv_append_fp8 followed by
+ * mcpu_paged_attention_forward_fp8 (decode rows; same rules and results)
+ * per slice, with the same host buffers, slicing, copies and errors. */
+mcpu_status mcpu_paged_attention_host_fp8(mcpu_host_stage* stage, const void* q_host, const void* k_new_host,
+                                          const void* v_new_host, void* kv8, const int32_t* block_table,
+                                          const int32_t* seq_lens_host, const int32_t* query_start_loc_host,
+                                          int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
+                                          void* out_host, float* lse_host, void* workspace, size_t workspace_bytes,
+                                          const mcpu_options* opts, int32_t slices, mcpu_stream_t stream);
 /* The row ranges mcpu_paged_attention_host uses for `slices` > 0 slices:
  * writes row_begin[0 .. n] (row_begin[0] = 0, row_begin[n] = num_seqs,
  * strictly increasing) and returns the number n of non-empty slices (0 for

@@ -190,13 +190,29 @@ int32_t mcpu_host_slice_rows(const int32_t* query_start_loc_host, int32_t num_se
   return n;
 }
 
-mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, const void* k_new_host,
-                                      const void* v_new_host, void* k_cache, void* v_cache,
-                                      const int32_t* block_table, const int32_t* seq_lens_host,
-                                      const int32_t* query_start_loc_host, int32_t sliding_window,
-                                      float softmax_scale, const mcpu_dims* dims, void* out_host, float* lse_host,
-                                      void* workspace, size_t workspace_bytes, const mcpu_options* opts,
-                                      int32_t slices, mcpu_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// The device-side arguments of one slice: its rows' block-table rows,
+// seq_lens and rebased query_start_loc, and its tokens' staging.
+struct Slice {
+  mcpu_dims dims;
+  const int32_t *block_table, *seq_lens, *query_start_loc;
+  const void *q, *k_new, *v_new;
+  void* out;
+  float* lse;
+};
+
+// The pipeline shared by the bf16 and fp8 calls: checks, slicing, the
+// copies in and out on the stage's streams, and `compute(slice)` (the KV
+// append and forward of one slice, enqueued on `stream`) in between.
+template <typename Compute>
+mcpu_status host_call(mcpu_host_stage* hs, const void* q_host, const void* k_new_host, const void* v_new_host,
+                      const int32_t* block_table, const int32_t* seq_lens_host,
+                      const int32_t* query_start_loc_host, float softmax_scale, const mcpu_dims* dims,
+                      void* out_host, float* lse_host, void* workspace, size_t workspace_bytes, int32_t slices,
+                      mcpu_stream_t stream, Compute compute) {
   if (!hs || !dims || !seq_lens_host || !query_start_loc_host) return MCPU_ERR_INVALID_ARG;
   if (!on_stage_device(hs)) return MCPU_ERR_INVALID_ARG;
   const int32_t B = dims->num_seqs, T = dims->total_q;
@@ -214,8 +230,7 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
   if (need == 0) return MCPU_ERR_UNSUPPORTED;
   if (!workspace || workspace_bytes < need) return workspace ? MCPU_ERR_WORKSPACE_TOO_SMALL : MCPU_ERR_INVALID_ARG;
   if (T == 0 || B == 0) return MCPU_OK;
-  if (!q_host || !k_new_host || !v_new_host || !out_host || !lse_host || !k_cache || !v_cache || !block_table)
-    return MCPU_ERR_INVALID_ARG;
+  if (!q_host || !k_new_host || !v_new_host || !out_host || !lse_host || !block_table) return MCPU_ERR_INVALID_ARG;
 
   const int64_t q_row = (int64_t)dims->num_q_heads * kRowBytes, kv_row = (int64_t)dims->num_kv_heads * kRowBytes;
   const int64_t lse_row = (int64_t)dims->num_q_heads * 4;
@@ -260,18 +275,19 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
     if (e == cudaSuccess) e = cudaStreamWaitEvent(s, hs->ev_in[k], 0);
     if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
     // the slice's KV append and forward on the caller's stream
-    mcpu_dims d = *dims;
-    d.num_seqs = b - a;
-    d.total_q = (int32_t)nt;
-    const int32_t* bt = block_table + (int64_t)a * dims->max_pages_per_seq;
-    const int32_t* qsl = sl.qsl + a + k;
-    mcpu_status st = mcpu_kv_append(sl.kn + t0 * kv_row, sl.vn + t0 * kv_row, k_cache, v_cache, bt, sl.sl + a, qsl,
-                                    &d, static_cast<int32_t*>(workspace), stream);
-    if (st != MCPU_OK) return fail_after_enqueue(hs, sl, s, st);
-    st = mcpu_paged_attention_forward(sl.q + t0 * q_row, k_cache, v_cache, bt, sl.sl + a, qsl, sliding_window,
-                                      softmax_scale, &d, sl.out + t0 * q_row,
-                                      reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sl.lse) + t0 * lse_row),
-                                      workspace, workspace_bytes, opts, stream);
+    Slice c;
+    c.dims = *dims;
+    c.dims.num_seqs = b - a;
+    c.dims.total_q = (int32_t)nt;
+    c.block_table = block_table + (int64_t)a * dims->max_pages_per_seq;
+    c.seq_lens = sl.sl + a;
+    c.query_start_loc = sl.qsl + a + k;
+    c.q = sl.q + t0 * q_row;
+    c.k_new = sl.kn + t0 * kv_row;
+    c.v_new = sl.vn + t0 * kv_row;
+    c.out = sl.out + t0 * q_row;
+    c.lse = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sl.lse) + t0 * lse_row);
+    const mcpu_status st = compute(c);
     if (st != MCPU_OK) return fail_after_enqueue(hs, sl, s, st);
     // its outputs, once computed
     e = cudaEventRecord(hs->ev_done[k], s);
@@ -288,6 +304,51 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
   if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
   hs->any_out = true;
   return MCPU_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, const void* k_new_host,
+                                      const void* v_new_host, void* k_cache, void* v_cache,
+                                      const int32_t* block_table, const int32_t* seq_lens_host,
+                                      const int32_t* query_start_loc_host, int32_t sliding_window,
+                                      float softmax_scale, const mcpu_dims* dims, void* out_host, float* lse_host,
+                                      void* workspace, size_t workspace_bytes, const mcpu_options* opts,
+                                      int32_t slices, mcpu_stream_t stream) {
+  if (!k_cache || !v_cache) return MCPU_ERR_INVALID_ARG;
+  int32_t* status = static_cast<int32_t*>(workspace);
+  return host_call(hs, q_host, k_new_host, v_new_host, block_table, seq_lens_host, query_start_loc_host,
+                   softmax_scale, dims, out_host, lse_host, workspace, workspace_bytes, slices, stream,
+                   [&](const Slice& c) {
+                     mcpu_status st = mcpu_kv_append(c.k_new, c.v_new, k_cache, v_cache, c.block_table, c.seq_lens,
+                                                     c.query_start_loc, &c.dims, status, stream);
+                     if (st != MCPU_OK) return st;
+                     return mcpu_paged_attention_forward(c.q, k_cache, v_cache, c.block_table, c.seq_lens,
+                                                         c.query_start_loc, sliding_window, softmax_scale, &c.dims,
+                                                         c.out, c.lse, workspace, workspace_bytes, opts, stream);
+                   });
+}
+
+mcpu_status mcpu_paged_attention_host_fp8(mcpu_host_stage* hs, const void* q_host, const void* k_new_host,
+                                          const void* v_new_host, void* kv8, const int32_t* block_table,
+                                          const int32_t* seq_lens_host, const int32_t* query_start_loc_host,
+                                          int32_t sliding_window, float softmax_scale, const mcpu_dims* dims,
+                                          void* out_host, float* lse_host, void* workspace, size_t workspace_bytes,
+                                          const mcpu_options* opts, int32_t slices, mcpu_stream_t stream) {
+  if (!kv8) return MCPU_ERR_INVALID_ARG;
+  int32_t* status = static_cast<int32_t*>(workspace);
+  return host_call(hs, q_host, k_new_host, v_new_host, block_table, seq_lens_host, query_start_loc_host,
+                   softmax_scale, dims, out_host, lse_host, workspace, workspace_bytes, slices, stream,
+                   [&](const Slice& c) {
+                     mcpu_status st = mcpu_kv_append_fp8(c.k_new, c.v_new, kv8, c.block_table, c.seq_lens,
+                                                         c.query_start_loc, &c.dims, status, stream);
+                     if (st != MCPU_OK) return st;
+                     return mcpu_paged_attention_forward_fp8(c.q, kv8, c.block_table, c.seq_lens, c.query_start_loc,
+                                                             sliding_window, softmax_scale, &c.dims, c.out, c.lse,
+                                                             workspace, workspace_bytes, opts, stream);
+                   });
 }
 
 }  // extern "C"

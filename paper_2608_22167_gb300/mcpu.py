@@ -131,6 +131,11 @@ _lib.mcpu_paged_attention_host.argtypes = [
     ctypes.c_size_t, ctypes.POINTER(Options), ctypes.c_int32, _P,
 ]
 _lib.mcpu_paged_attention_host.restype = ctypes.c_int
+_lib.mcpu_paged_attention_host_fp8.argtypes = [
+    _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P,
+    ctypes.c_size_t, ctypes.POINTER(Options), ctypes.c_int32, _P,
+]
+_lib.mcpu_paged_attention_host_fp8.restype = ctypes.c_int
 
 MAX_HOST_SLICES = 8
 MAX_HOST_SLOTS = 4
@@ -429,5 +434,27 @@ def mcpu_paged_attention_host(stage, q_host, k_new_host, v_new_host, k_cache, v_
             ctypes.byref(opts), int(slices), _stream(stream),
         ),
         "mcpu_paged_attention_host",
+    )
+    stage._pending.append((q_host, k_new_host, v_new_host, out_host, lse_host, sl, qsl, opts))
+
+
+def mcpu_paged_attention_host_fp8(stage, q_host, k_new_host, v_new_host, kv8, block_table, seq_lens_host,
+                                  query_start_loc_host, sliding_window, softmax_scale, out_host, lse_host, workspace,
+                                  flags=0, split_pages=0, slices=0, stream=None, sinks=None):
+    """mcpu_paged_attention_host over an fp8 pool kv8 [P, Hkv, 2176] (decode rows)."""
+    for t in (q_host, k_new_host, v_new_host, out_host, lse_host):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError("q / k_new / v_new / out / lse must be contiguous host tensors")
+    sl, qsl = _host_i32(seq_lens_host), _host_i32(query_start_loc_host)
+    d = dims_fp8(q_host, kv8, block_table, sl)
+    opts = _options(d.num_q_heads, flags, split_pages, None, sinks)
+    _check(
+        _lib.mcpu_paged_attention_host_fp8(
+            stage.handle, _ptr(q_host), _ptr(k_new_host), _ptr(v_new_host), _ptr(kv8), _ptr(block_table), _ptr(sl),
+            _ptr(qsl), int(sliding_window), float(softmax_scale), ctypes.byref(d), _ptr(out_host), _ptr(lse_host),
+            _ptr(workspace), int(workspace.numel() * workspace.element_size()), ctypes.byref(opts), int(slices),
+            _stream(stream),
+        ),
+        "mcpu_paged_attention_host_fp8",
     )
     stage._pending.append((q_host, k_new_host, v_new_host, out_host, lse_host, sl, qsl, opts))

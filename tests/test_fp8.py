@@ -289,6 +289,35 @@ def test_long_batch_sampled_at_full_size():
     assert_parity(go, gl, oracle.bf16_bits_to_float(ro), rl, "long_b512 fp8")
 
 
+@pytest.mark.parametrize("slices", [1, 3])
+@pytest.mark.parametrize("seed", range(3))
+def test_host_buffer_call(seed, slices):
+    # mcpu_paged_attention_host_fp8: q / k_new / v_new / out / lse in host memory
+    b = _decode_batch(3700 + seed, B=9, window=(0, 128, 0)[seed])
+    run = Fp8Run(b)
+    lay = b.layers[0]
+    pin = lambda t: t.cpu().contiguous().pin_memory()  # noqa: E731
+    qh, knh, vnh = pin(lay.q), pin(lay.k_new), pin(lay.v_new)
+    slh = torch.from_numpy(b.seq_lens).to(torch.int32)
+    qslh = torch.from_numpy(b.query_start_loc).to(torch.int32)
+    out_h = torch.full(qh.shape, float("nan"), dtype=torch.bfloat16).pin_memory()
+    lse_h = torch.full(qh.shape[:2], float("nan"), dtype=torch.float32).pin_memory()
+    st = mcpu.HostStage(qh.shape[0], b.num_seqs, b.num_q_heads, b.num_kv_heads)
+    mcpu.mcpu_paged_attention_host_fp8(st, qh, knh, vnh, run.kv8, run.bt, slh, qslh, run.window, b.softmax_scale,
+                                       out_h, lse_h, run.ws, slices=slices)
+    mcpu.mcpu_host_stage_sync(st)
+    code, bits = run.status()
+    assert code == 0, f"device status bits {bits}"
+    pools = run.oracle_append()
+    for g, r, what in zip(run.pools_host(), pools, ("k codes", "v codes", "k scales", "v scales")):
+        assert np.array_equal(np.ascontiguousarray(g).view(np.uint8), np.ascontiguousarray(r).view(np.uint8)), what
+    h = run.h
+    ro, rl = oracle.paged_attention_fp8(h["q"], *pools, h["block_table"], h["seq_lens"], h["query_start_loc"],
+                                        h["sliding_window"], h["softmax_scale"])
+    assert_parity(out_h.float().numpy(), lse_h.numpy(), oracle.bf16_bits_to_float(ro), rl, f"host fp8 {seed}")
+    st.close()
+
+
 def test_fp8_and_bf16_paths_agree_on_exactly_representable_pools():
     # pools whose bf16 values are e4m3 codes times power-of-two row scales:
     # both storage formats describe the same K and V
