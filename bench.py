@@ -632,7 +632,18 @@ def run_ours(args, rank, world, dev):
                     "kernel": "append_tc_kernel",
                     "peak_source": f"{peak_src} bf16_tflops (burst)", "ms_per_step": round(app_ms, 4)}
     cands = [r for r in (roof_dec, roof_app) if r is not None]
-    dominant = max(cands, key=lambda r: r["ms_per_step"]) if cands else None
+    # the kernel that bounds the step: the tensor-core append kernel when the
+    # step's flops take longer at the bf16 peak than its KV bytes at the HBM
+    # peak (the decode kernels' spans on the side stream then include time
+    # spent waiting for SMs the append kernel holds), else the decode kernel
+    step_flops = sum(s["flops"] for s in per_layer)
+    tensor_bound = step_flops / (tc_burst * 1e12) > sum(s["kv_bytes"] for s in per_layer) / (hbm * 1e9)
+    if tensor_bound and roof_app is not None:
+        dominant = roof_app
+    elif roof_dec is not None:
+        dominant = roof_dec
+    else:
+        dominant = max(cands, key=lambda r: r["ms_per_step"]) if cands else None
 
     # ---- end to end: host buffers, copies inside the timed region: every
     # layer through mcpu_paged_attention_host (_fp8 over fp8 pools), which
