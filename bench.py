@@ -84,14 +84,17 @@ APPEND_TC_SOURCES = [
     "paper_2608_22167_gb300/csrc/append_tc.cu",
     "paper_2608_22167_gb300/csrc/tcgen05.cuh",
     "paper_2608_22167_gb300/csrc/common.cuh",
+    "paper_2608_22167_gb300/csrc/plan.cu",  # item order and split lengths shape the traffic
 ]
 DECODE_SOURCES = [
     "paper_2608_22167_gb300/csrc/decode.cu",
     "paper_2608_22167_gb300/csrc/common.cuh",
+    "paper_2608_22167_gb300/csrc/plan.cu",
 ]
 FP8_SOURCES = [
     "paper_2608_22167_gb300/csrc/fp8.cu",
     "paper_2608_22167_gb300/csrc/common.cuh",
+    "paper_2608_22167_gb300/csrc/plan.cu",
 ]
 FP8_WORKLOADS = ("tiny", "decode", "long")
 NOMINAL_HBM_GBS = 8000.0  # the nominal HBM3e figure the targets are also quoted against
