@@ -378,6 +378,27 @@ mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream,
 /* Enqueues a clear of the workspace status word on `stream`. */
 mcpu_status mcpu_reset_device_status(void* workspace, mcpu_stream_t stream);
 
+/* Self-check of the device-side timeout path (no counterpart in the paper:
+ * it exists so that the path can be exercised on a GPU without a fault or a
+ * hang). Every wait in the kernels above is bounded by the library's wait
+ * limit (200 ms of the GPU's global timer); when one runs out, the kernel
+ * sets the timeout bit of the status word and returns, and
+ * mcpu_read_device_status reports MCPU_ERR_TIMEOUT. Inputs cannot cause
+ * that, so this call enqueues one small kernel (one CTA) on `stream` in
+ * which a warp waits, with the same bounded wait as the decode kernels, on
+ * a shared-memory barrier that nothing ever completes, and a second warp on
+ * one that does complete. It runs for about the wait limit.
+ *   workspace  device memory; only its first 4 bytes (the status word) are
+ *              touched: the timeout bit is OR-ed in if the wait gave up.
+ *   report     device memory, int64_t[4], 8-byte aligned, written:
+ *              [0] 1 if the completing wait returned success, else 0;
+ *              [1] 1 if the never-completing wait returned success (a
+ *                  failure of the check), else 0;
+ *              [2] nanoseconds that wait took; [3] the wait limit in ns.
+ * Returns MCPU_ERR_INVALID_ARG for null or misaligned pointers and
+ * MCPU_ERR_CUDA if the launch fails; otherwise MCPU_OK (asynchronous). */
+mcpu_status mcpu_selftest_wait_timeout(void* workspace, int64_t* report, mcpu_stream_t stream);
+
 /* Static, human-readable name of a status code. */
 const char* mcpu_status_string(mcpu_status status);
 

@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libmcpu.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["api.cu", "api_noalloc.cu", "api_host.cu", "plan.cu", "decode.cu", "append_attn.cu", "append_tc.cu", "merge.cu",
-           "kv_append.cu", "rope_append.cu", "fp8.cu"]
+           "kv_append.cu", "rope_append.cu", "fp8.cu", "selftest.cu"]
 
 
 def nvcc() -> str:

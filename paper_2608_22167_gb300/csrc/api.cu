@@ -166,7 +166,7 @@ mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : cuda_
 
 extern "C" {
 
-int32_t mcpu_abi_version(void) { return 4; }
+int32_t mcpu_abi_version(void) { return 5; }
 
 int32_t mcpu_last_cuda_error(void) { return t_last_cuda_error; }
 

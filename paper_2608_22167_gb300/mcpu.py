@@ -109,6 +109,8 @@ _lib.mcpu_read_device_status.argtypes = [_P, _P, ctypes.POINTER(ctypes.c_int32)]
 _lib.mcpu_read_device_status.restype = ctypes.c_int
 _lib.mcpu_reset_device_status.argtypes = [_P, _P]
 _lib.mcpu_reset_device_status.restype = ctypes.c_int
+_lib.mcpu_selftest_wait_timeout.argtypes = [_P, _P, _P]
+_lib.mcpu_selftest_wait_timeout.restype = ctypes.c_int
 _lib.mcpu_status_string.argtypes = [ctypes.c_int]
 _lib.mcpu_status_string.restype = ctypes.c_char_p
 _lib.mcpu_abi_version.argtypes = []
@@ -339,6 +341,17 @@ def mcpu_read_device_status(workspace, stream=None):
 
 def mcpu_reset_device_status(workspace, stream=None):
     _check(_lib.mcpu_reset_device_status(_ptr(workspace), _stream(stream)), "mcpu_reset_device_status")
+
+
+def mcpu_selftest_wait_timeout(workspace, report, stream=None):
+    """Enqueues the timeout self-check: ``report`` is a device int64 tensor of
+    4 entries (completing wait ok, never-completing wait ok, its duration in
+    ns, the wait limit in ns); the status word of ``workspace`` gets the
+    timeout bit when the wait gives up."""
+    if report.dtype != torch.int64 or report.numel() < 4 or not report.is_contiguous():
+        raise McpuError(1, "mcpu_selftest_wait_timeout")
+    _check(_lib.mcpu_selftest_wait_timeout(_ptr(workspace), _ptr(report), _stream(stream)),
+           "mcpu_selftest_wait_timeout")
 
 
 def new_workspace(d: Dims, device="cuda") -> torch.Tensor:

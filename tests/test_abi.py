@@ -152,6 +152,16 @@ def test_status_strings(lib):
         seen.add(s)
 
 
+def test_timeout_selftest_host_checks(lib):
+    f = _fn(lib, "mcpu_selftest_wait_timeout")
+    f.argtypes = [ctypes.c_void_p] * 3
+    P = 1 << 20
+    assert f(None, P, None) == 1
+    assert f(P, None, None) == 1
+    assert f(P + 2, P, None) == 1  # status word not 4-byte aligned
+    assert f(P, P + 4, None) == 1  # report not 8-byte aligned
+
+
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-GPU error path")
 def test_no_gpu_is_a_clean_error(lib):
     fwd = _fn(lib, "mcpu_paged_attention_forward")
