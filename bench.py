@@ -58,6 +58,8 @@ WORKLOAD_DESC = {
     "rollout": "rollout step: 24 layers alternating SWA-128/full, 48 GRPO groups x 8 rows sharing prompt "
                "pages (prompt U[1024,8192], continuation U[0,24576]), 15% append rows (logU[64,1024]), "
                "64q/8kv, D=64, page 16, bf16",
+    "rollout_small": "rollout step at 8 GRPO groups x 8 rows and 4 layers (SWA-128/full alternating), same "
+                     "distributions; profiling case",
 }
 
 
@@ -355,7 +357,7 @@ class Fp8Stepper(Stepper):
 def make_batch(name, dev, rank):
     fn = W.CONFIGS[name]
     seed = {"tiny": 1001, "decode": 1002, "mixed": 1003, "mixed_small": 1013, "long": 1004,
-            "rollout": 1005}[name] + 7 * rank
+            "rollout": 1005, "rollout_small": 1015}[name] + 7 * rank
     return fn(seed=seed, device=dev)
 
 

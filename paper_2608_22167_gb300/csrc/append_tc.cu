@@ -83,11 +83,27 @@ namespace {
 
 // Bounded wait that also gives up when another role has aborted. The polls
 // sleep (the producer and the MMA issuers wait most of the time and share
-// sub-partitions with the softmax warps).
+// sub-partitions with the softmax warps). Used by the producer and issuers.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int32_t* abort_flag) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (!mbar_try_wait_sleep(bar, parity, 10000)) {
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > kWaitTimeoutNs) {
+      *abort_flag = 1;
+      return false;
+    }
+  }
+  return true;
+}
+
+// The softmax warps' bounded wait: the same, with plain polls (no
+// suspend-time hint). The softmax is the critical path and rarely waits
+// long; a sleeping poll there made the mixed batch's step ~0.65 % slower.
+__device__ __forceinline__ bool wait_bar_poll(uint32_t bar, uint32_t parity, volatile int32_t* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
     if (*abort_flag) return false;
     if (global_timer_ns() - t0 > kWaitTimeoutNs) {
       *abort_flag = 1;
@@ -411,7 +427,7 @@ __global__ void __maxnreg__(144)
     bool ok = true;
     for (int i = 0; ok; ++i) {
       const int slot = i & 1;
-      ok = __all_sync(0xffffffffu, wait_bar(bar(st.item_full[slot]), (i >> 1) & 1, abort_flag));
+      ok = __all_sync(0xffffffffu, wait_bar_poll(bar(st.item_full[slot]), (i >> 1) & 1, abort_flag));
       if (!ok) break;
       const int idx = st.item_idx[slot];
       const AppendItem a = st.items[slot];
@@ -429,7 +445,7 @@ __global__ void __maxnreg__(144)
       const int wp_max = a.pos_begin + min(x * tile_tok + (wq * 32 + 31) / g, last_tok);
       float m_ref = -INFINITY, l = 0.f;
       for (int b = 0; b < nb; ++b, ++blk) {
-        ok = __all_sync(0xffffffffu, wait_bar(bar(st.s_full[x]), blk & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, wait_bar_poll(bar(st.s_full[x]), blk & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
         const int kb = kb0 + b * kTcKeys;
@@ -443,7 +459,7 @@ __global__ void __maxnreg__(144)
         float l0 = chunk_probs(sv, p.scale_log2, m_ref, alpha, pk);
         // the single P buffer was last read by PV_X(blk - 1)
         if (blk >= 1) {
-          ok = __all_sync(0xffffffffu, wait_bar(bar(st.o_ready[x]), (blk - 1) & 1, abort_flag));
+          ok = __all_sync(0xffffffffu, wait_bar_poll(bar(st.o_ready[x]), (blk - 1) & 1, abort_flag));
           if (!ok) break;
           tc_fence_after();
         }
@@ -495,7 +511,7 @@ __global__ void __maxnreg__(144)
       if (!ok) break;
       // epilogue: the last PV_X of the item
       if (nb > 0) {
-        ok = __all_sync(0xffffffffu, wait_bar(bar(st.o_ready[x]), (blk - 1) & 1, abort_flag));
+        ok = __all_sync(0xffffffffu, wait_bar_poll(bar(st.o_ready[x]), (blk - 1) & 1, abort_flag));
         if (!ok) break;
       }
       tc_fence_after();

@@ -304,7 +304,7 @@ def rollout_lengths(seed=1005, groups=48, group_size=8, append_frac=0.15):
     return S, L, group_of_row, prompt, shared
 
 
-def config_rollout(seed=1005, device="cpu", layers=24, window=128, groups=48) -> Batch:
+def config_rollout(seed=1005, device="cpu", layers=24, window=128, groups=48, name=None) -> Batch:
     """Full rollout step: ``layers`` layers alternating sliding-window-128
     (even) and full-context (odd) attention over 48 GRPO groups x 8 rows.
     Full-context layers share one pool in which every group's full prompt
@@ -313,7 +313,7 @@ def config_rollout(seed=1005, device="cpu", layers=24, window=128, groups=48) ->
     S, L, grp, prompt, shared = rollout_lengths(seed, groups=groups)
     wins = [window if (i % 2 == 0) else 0 for i in range(layers)]
     b = build_batch(
-        "rollout_g48x8",
+        name or f"rollout_g{groups}x8",
         seed,
         S,
         L,
@@ -340,6 +340,13 @@ def config_mixed_small(seed=1013, device="cpu") -> Batch:
     return build_batch("mixed_b64", seed, prior + L, L, 64, 8, device=device)
 
 
+def config_rollout_small(seed=1015, device="cpu") -> Batch:
+    """The rollout step's distributions at 8 GRPO groups (64 rows, 10
+    appending) and 4 layers (window, full, window, full): a profiling case
+    for the window and full-context layers' kernels whose pools stay small."""
+    return config_rollout(seed=seed, device=device, layers=4, groups=8, name="rollout_g8x8_l4")
+
+
 CONFIGS = {
     "tiny": config_tiny,
     "decode": config_decode,
@@ -347,6 +354,7 @@ CONFIGS = {
     "mixed_small": config_mixed_small,
     "long": config_long,
     "rollout": config_rollout,
+    "rollout_small": config_rollout_small,
 }
 
 
