@@ -19,7 +19,8 @@ per token. Attended tokens/s (sum over queries of visible keys) is reported
 beside it.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload mixed|decode|long|rollout|tiny]
+                  [--workload mixed|decode|long|rollout|tiny|mixed_small|rollout_small|churn]
+                  [--kv bf16|fp8] [--launch graph|eager]
 
 Prints one JSON line (rank 0). Under torchrun each rank runs an independent
 replica on its own GPU (the path has no exchange step); value is the total
