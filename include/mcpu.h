@@ -46,6 +46,10 @@
  *                 block is page_size * D * 2 contiguous bytes.
  *   block_table   [B, max_pages_per_seq] int32: logical page -> physical page.
  *                 Entries no query can see may hold anything (e.g. -1).
+ *                 Slots of a page that no query of the call can see (never
+ *                 written yet, or before a window) may hold anything, NaN
+ *                 and Inf included: the kernels give them no weight and zero
+ *                 their V rows before the weighted sum.
  *   seq_lens      [B] int32;  query_start_loc [B + 1] int32 (prefix sums, [0] = 0)
  *   out           [T, H_q, D] bf16;  lse [T, H_q] float (natural log of the
  *                 softmax normaliser sum_j exp(scale * q.k_j); -inf if empty)
@@ -126,7 +130,10 @@ typedef struct mcpu_options {
 size_t mcpu_workspace_size(const mcpu_dims* dims);
 
 /*
- * KV append (the new tokens of every row enter the cache).
+ * KV append (the new tokens of every row enter the cache): the step between
+ * two generations of a trajectory in which the tool observation's tokens (an
+ * append row) or the token just generated (a decode row) join its context
+ * (paper §3.2, the run stage's alternation of generation and tool calls).
  * For each row r and i < L_r, copies k_new[query_start_loc[r] + i] (all kv
  * heads) bit for bit to k_cache[block_table[r][pos / page]][h][pos % page]
  * with pos = S_r - L_r + i; likewise v_new into v_cache. Decode rows append
@@ -142,7 +149,11 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
 /*
  * Paged attention forward over a mixed batch of decode rows (L_r = 1) and
  * append rows (L_r > 1, causal within the chunk), with an optional sliding
- * window (W <= 0: full context). Rows with L_r = 0 produce nothing.
+ * window (W <= 0: full context). This is the attention of the generation
+ * that bounds the run stage (paper §3.2; again §4.2): hundreds of
+ * trajectories in flight, each either generating one token or taking in a
+ * tool observation, the n = 8 samples of a GRPO task sharing their prompt
+ * (§4; App. B, Tab. "hparams"), sequences up to 128k tokens. Rows with L_r = 0 produce nothing.
  * softmax_scale (> 0, finite) multiplies q.k (1/sqrt(D) for gpt-oss). Rows that are
  * adjacent in the batch and whose block tables start with the same physical
  * pages (a GRPO group's shared prompt) are detected on the device and their
@@ -378,6 +389,38 @@ mcpu_status mcpu_read_device_status(const void* workspace, mcpu_stream_t stream,
 /* Enqueues a clear of the workspace status word on `stream`. */
 mcpu_status mcpu_reset_device_status(void* workspace, mcpu_stream_t stream);
 
+/* Self-check of the append kernel's abort path (no counterpart in the paper:
+ * it exercises, on a GPU and without a fault or a hang, what the tcgen05
+ * append kernel does when one of its waits runs out). Runs the planner and
+ * then the self-test form of that kernel as ONE CTA over the batch given
+ * (same arguments and rules as mcpu_paged_attention_forward; no window, no
+ * options; the batch needs an append row whose first work item spans at
+ * least two 128-key blocks). In that form one role, chosen by stall_role,
+ * stops at the second key block of its first item and waits, for half the
+ * library's wait limit, on a barrier nothing completes:
+ *   0  the softmax warps of the first query tile,
+ *   1  the TMA producer warp,
+ *   2  the MMA issuer of the first query tile.
+ * It then raises the CTA's abort flag with its own mark (2); every other
+ * role, waiting with the full limit, must leave its wait on seeing the flag
+ * (a role whose own wait ran out would overwrite the mark with 1, half a
+ * limit later), the MMA issuers wait for their MMAs in flight and the
+ * producer for its copies in flight, and TMEM is freed. Outputs of the rows
+ * are undefined afterwards; the workspace status word gets the timeout bit.
+ *   report  device memory, int64_t[16], 8-byte aligned, cleared and written:
+ *           [0] the abort flag at the end (2 when only the stalled role ran
+ *               out of its wait); [1 + w] nanoseconds from kernel start to
+ *               the moment warp w (0..10) left its role; [12] the stalled
+ *               wait in ns; [13] the library's wait limit in ns; [14] 1 once
+ *               TMEM was freed; [15] unused.
+ * Returns MCPU_ERR_INVALID_ARG for a bad role, null or misaligned pointers
+ * or an empty batch; otherwise the forward call's errors (asynchronous). */
+mcpu_status mcpu_selftest_append_abort(const void* q, const void* k_cache, const void* v_cache,
+                                       const int32_t* block_table, const int32_t* seq_lens,
+                                       const int32_t* query_start_loc, float softmax_scale, const mcpu_dims* dims,
+                                       void* out, float* lse, void* workspace, size_t workspace_bytes,
+                                       int32_t stall_role, int64_t* report, mcpu_stream_t stream);
+
 /* Self-check of the device-side timeout path (no counterpart in the paper:
  * it exists so that the path can be exercised on a GPU without a fault or a
  * hang). Every wait in the kernels above is bounded by the library's wait
@@ -403,9 +446,11 @@ mcpu_status mcpu_selftest_wait_timeout(void* workspace, int64_t* report, mcpu_st
 const char* mcpu_status_string(mcpu_status status);
 
 /* The cudaError_t (as an integer) of the most recent CUDA call that failed
- * inside mcpu_kv_append or mcpu_paged_attention_forward on the calling
- * thread, i.e. the cause behind their last MCPU_ERR_CUDA; 0 if none has
- * failed. Not cleared by later successful calls. */
+ * inside an entry point of this library (mcpu_kv_append,
+ * mcpu_paged_attention_forward, mcpu_paged_attention_forward_noalloc and the
+ * others) on the calling thread, i.e. the cause behind its last
+ * MCPU_ERR_CUDA; 0 if none has failed. Not cleared by later successful
+ * calls. */
 int32_t mcpu_last_cuda_error(void);
 
 /* Version of this ABI (bumped on any signature change or addition). */

@@ -8,6 +8,7 @@
 #include <mutex>
 
 #include "../../include/mcpu.h"
+#include "api_internal.h"
 #include "common.cuh"
 
 namespace mcpu {
@@ -21,6 +22,8 @@ cudaError_t launch_append(const CUtensorMap& kmap, const CUtensorMap& vmap, cons
 cudaError_t prepare_append_kernel(int* bpsm);
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                              const AttnParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_append_tc_selftest(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
+                                      const AttnParams& p, cudaStream_t stream);
 cudaError_t prepare_append_tc_kernel(int* bpsm);
 cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream);
 cudaError_t prepare_merge_kernel();
@@ -64,14 +67,6 @@ struct DeviceState {
 
 std::mutex g_mu;
 DeviceState g_dev[kMaxDevices];
-
-// most recent failing CUDA call of this thread's entry-point calls
-thread_local int32_t t_last_cuda_error = 0;
-
-mcpu_status cuda_fail(cudaError_t e) {
-  t_last_cuda_error = (int32_t)e;
-  return MCPU_ERR_CUDA;
-}
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
@@ -143,7 +138,18 @@ bool encode_query(CUtensorMap* map, const void* q, int32_t total_q, int32_t num_
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Checks shared by both entry points. Returns MCPU_OK or the error.
+}  // namespace
+
+namespace mcpu {
+
+// most recent failing CUDA call of this thread's entry-point calls
+thread_local int32_t t_last_cuda_error = 0;
+
+mcpu_status cuda_fail(cudaError_t e) {
+  t_last_cuda_error = (int32_t)e;
+  return MCPU_ERR_CUDA;
+}
+
 mcpu_status check_dims(const mcpu_dims* d) {
   if (!d) return MCPU_ERR_INVALID_ARG;
   if (d->num_seqs < 0 || d->total_q < 0 || d->max_pages_per_seq < 0 || d->num_pages < 0 || d->num_q_heads <= 0 ||
@@ -162,13 +168,13 @@ mcpu_status check_dims(const mcpu_dims* d) {
 
 mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : cuda_fail(e); }
 
-}  // namespace
+}  // namespace mcpu
 
 extern "C" {
 
-int32_t mcpu_abi_version(void) { return 5; }
+int32_t mcpu_abi_version(void) { return 6; }
 
-int32_t mcpu_last_cuda_error(void) { return t_last_cuda_error; }
+int32_t mcpu_last_cuda_error(void) { return mcpu::t_last_cuda_error; }
 
 const char* mcpu_status_string(mcpu_status s) {
   switch (s) {
@@ -466,6 +472,68 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
     e = launch_merge(p, grid, s);
   }
   if (e == cudaSuccess) e = mark(5);
+  return from_cuda(e);
+}
+
+mcpu_status mcpu_selftest_append_abort(const void* q, const void* k_cache, const void* v_cache,
+                                       const int32_t* block_table, const int32_t* seq_lens,
+                                       const int32_t* query_start_loc, float softmax_scale, const mcpu_dims* dims,
+                                       void* out, float* lse, void* workspace, size_t workspace_bytes,
+                                       int32_t stall_role, int64_t* report, mcpu_stream_t stream) {
+  mcpu_status st = check_dims(dims);
+  if (st != MCPU_OK) return st;
+  if (stall_role < 0 || stall_role > 2) return MCPU_ERR_INVALID_ARG;
+  if (!report || !aligned(report, 8)) return MCPU_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.f) || softmax_scale > 3.0e38f) return MCPU_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256)) return MCPU_ERR_INVALID_ARG;
+  if (workspace_bytes < mcpu_workspace_size(dims)) return MCPU_ERR_WORKSPACE_TOO_SMALL;
+  if (dims->total_q == 0 || dims->num_seqs == 0) return MCPU_ERR_INVALID_ARG;
+  if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !query_start_loc || !out || !lse)
+    return MCPU_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) || !aligned(lse, 4) ||
+      !aligned(block_table, 4) || !aligned(seq_lens, 4) || !aligned(query_start_loc, 4))
+    return MCPU_ERR_INVALID_ARG;
+  if (dims->num_pages < 1 || dims->max_pages_per_seq < 1) return MCPU_ERR_INVALID_ARG;
+  DeviceState* dev = nullptr;
+  st = device_state(&dev);
+  if (st != MCPU_OK) return st;
+  const int64_t rows = (int64_t)dims->num_pages * dims->num_kv_heads * kPage;
+  const int group = dims->num_q_heads / dims->num_kv_heads;
+  CUtensorMap kmap, vmap, qmap;
+  if (!encode_pool(&kmap, k_cache, rows) || !encode_pool(&vmap, v_cache, rows) ||
+      !encode_query(&qmap, q, dims->total_q, dims->num_q_heads, group))
+    return MCPU_ERR_INVALID_ARG;
+  AttnParams p;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.block_table = block_table;
+  p.seq_lens = seq_lens;
+  p.qsl = query_start_loc;
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.lse = lse;
+  p.ws = static_cast<uint8_t*>(workspace);
+  p.num_seqs = dims->num_seqs;
+  p.total_q = dims->total_q;
+  p.max_pages = dims->max_pages_per_seq;
+  p.num_pages = dims->num_pages;
+  p.num_q_heads = dims->num_q_heads;
+  p.num_kv_heads = dims->num_kv_heads;
+  p.group = group;
+  p.lay = workspace_layout(p.num_seqs, p.total_q, p.num_q_heads, p.group);
+  p.window = 0;
+  p.scale_log2 = softmax_scale * 1.4426950408889634f;
+  p.total_warps_hint = dev->sms * dev->bpsm_decode * 4;
+  p.forced_split_pages = 0;
+  p.cascade_enabled = 0;
+  p.oob_row = (int32_t)rows;
+  p.append_tile_tok = kAppendTcRows / p.group;
+  p.sinks = nullptr;
+  p.decode_only = 0;
+  p.selftest_stall = stall_role;
+  p.selftest_report = report;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemsetAsync(report, 0, 16 * sizeof(int64_t), s);
+  if (e == cudaSuccess) e = launch_plan(p, s);
+  if (e == cudaSuccess) e = launch_append_tc_selftest(kmap, vmap, qmap, p, s);
   return from_cuda(e);
 }
 

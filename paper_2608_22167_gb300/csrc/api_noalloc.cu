@@ -20,6 +20,7 @@
 #include <mutex>
 
 #include "../../include/mcpu.h"
+#include "api_internal.h"
 #include "common.cuh"
 
 namespace mcpu {
@@ -59,25 +60,28 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 // kernels' shared-memory limits and occupancy.
 mcpu_status noalloc_device(NoallocDevice** out) {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MCPU_ERR_CUDA;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= kMaxDevices) return MCPU_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_mu);
   NoallocDevice& d = g_dev[dev];
   if (!d.ready) {
     if (!g_encode) {
       void* fn = nullptr;
       cudaDriverEntryPointQueryResult q;
-      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
-              cudaSuccess ||
-          q != cudaDriverEntryPointSuccess || fn == nullptr)
-        return MCPU_ERR_CUDA;
+      if ((e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q)) !=
+          cudaSuccess)
+        return cuda_fail(e);
+      if (q != cudaDriverEntryPointSuccess || fn == nullptr) return MCPU_ERR_CUDA;
       g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
     void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || ptr == nullptr) return MCPU_ERR_CUDA;
-    if (cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_plan_kernel() != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_decode_kernels(&d.bpsm_decode, &d.bpsm_cascade) != cudaSuccess) return MCPU_ERR_CUDA;
-    if (prepare_append_tc_kernel(&d.bpsm_append_tc) != cudaSuccess) return MCPU_ERR_CUDA;
+    if ((e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch)) != cudaSuccess) return cuda_fail(e);
+    if (ptr == nullptr) return MCPU_ERR_CUDA;
+    if ((e = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_plan_kernel()) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_decode_kernels(&d.bpsm_decode, &d.bpsm_cascade)) != cudaSuccess) return cuda_fail(e);
+    if ((e = prepare_append_tc_kernel(&d.bpsm_append_tc)) != cudaSuccess) return cuda_fail(e);
     if (d.bpsm_decode < 1 || d.bpsm_append_tc < 1) return MCPU_ERR_CUDA;
     d.scratch = ptr;
     d.ready = true;
@@ -103,17 +107,10 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
     const int32_t* query_start_loc, int32_t sliding_window, float softmax_scale, const mcpu_dims* dims, void* out,
     float* lse, int32_t* status_word, mcpu_stream_t stream) {
   // ---- the same argument checks as mcpu_paged_attention_forward
-  if (!dims) return MCPU_ERR_INVALID_ARG;
+  const mcpu_status dst = check_dims(dims);
+  if (dst != MCPU_OK) return dst;
   const mcpu_dims& d = *dims;
-  if (d.num_seqs < 0 || d.total_q < 0 || d.max_pages_per_seq < 0 || d.num_pages < 0 || d.num_q_heads <= 0 ||
-      d.num_kv_heads <= 0 || d.head_dim <= 0 || d.page_size <= 0 || d.num_q_heads % d.num_kv_heads != 0)
-    return MCPU_ERR_INVALID_ARG;
-  if (d.head_dim != kHeadDim || d.page_size != kPage) return MCPU_ERR_UNSUPPORTED;
   const int group = d.num_q_heads / d.num_kv_heads;
-  if (group != 1 && group != 2 && group != 4 && group != 8) return MCPU_ERR_UNSUPPORTED;
-  if (d.num_seqs > kMaxSeqs) return MCPU_ERR_UNSUPPORTED;
-  if ((int64_t)d.num_pages * d.num_kv_heads * kPage >= (int64_t)0x7fff0000) return MCPU_ERR_UNSUPPORTED;
-  if ((int64_t)d.max_pages_per_seq * kPage >= (int64_t)0x7fff0000) return MCPU_ERR_UNSUPPORTED;
   if (!(softmax_scale > 0.f) || softmax_scale > 3.0e38f) return MCPU_ERR_INVALID_ARG;
   // ---- the fixed scratch must hold the plan of this batch
   if (d.total_q > kNoallocMaxTokens) return MCPU_ERR_WORKSPACE_TOO_SMALL;
@@ -185,5 +182,5 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
   if (e == cudaSuccess) e = launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
   if (e == cudaSuccess && status_word)
     e = cudaMemcpyAsync(status_word, dev->scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s);
-  return e == cudaSuccess ? MCPU_OK : MCPU_ERR_CUDA;
+  return from_cuda(e);
 }

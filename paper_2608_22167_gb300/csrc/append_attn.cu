@@ -200,6 +200,12 @@ __global__ void __launch_bounds__(kAppWarps * 32)
       l0 = l0 * al0 + rs0;
       l1 = l1 * al1 + rs1;
 
+      // V rows of slots outside [key_begin, key_end) (the partial first page
+      // of a window, the partial last page) were perhaps never written and
+      // may hold NaN, which a zero weight does not cancel: they are zeroed in
+      // the operand. Per key step this lane's b0/b2 hold keys 2c, 2c + 1 and
+      // b1/b3 keys 2c + 8, 2c + 9 (c = lane & 3), the lower key in the low half.
+      const bool v_edge = kbase < a.key_begin || kbase + kKeyBlock > a.key_end;
       // O += P V, P from the S accumulators (key step ks covers keys 16ks..16ks+15)
 #pragma unroll
       for (int ks = 0; ks < 4; ++ks) {
@@ -207,10 +213,21 @@ __global__ void __launch_bounds__(kAppWarps * 32)
         const uint32_t pa1 = pack_bf16x2(sc[2 * ks][2], sc[2 * ks][3]);
         const uint32_t pa2 = pack_bf16x2(sc[2 * ks + 1][0], sc[2 * ks + 1][1]);
         const uint32_t pa3 = pack_bf16x2(sc[2 * ks + 1][2], sc[2 * ks + 1][3]);
+        uint32_t vm_lo = 0xffffffffu, vm_hi = 0xffffffffu;
+        if (v_edge) {
+          const int jv = kbase + ks * 16 + 2 * (lane & 3);
+          auto seen = [&](int j) { return j >= a.key_begin && j < a.key_end; };
+          vm_lo = (seen(jv) ? 0x0000ffffu : 0u) | (seen(jv + 1) ? 0xffff0000u : 0u);
+          vm_hi = (seen(jv + 8) ? 0x0000ffffu : 0u) | (seen(jv + 9) ? 0xffff0000u : 0u);
+        }
 #pragma unroll
         for (int dp = 0; dp < 4; ++dp) {
           uint32_t b0, b1, b2, b3;
           ldmatrix_x4_trans(vt + swz128(ks * 16 + ri + (mi & 1) * 8, 2 * dp + (mi >> 1)), b0, b1, b2, b3);
+          b0 &= vm_lo;
+          b2 &= vm_lo;
+          b1 &= vm_hi;
+          b3 &= vm_hi;
           mma_bf16_16816(o[2 * dp], pa0, pa1, pa2, pa3, b0, b1);
           mma_bf16_16816(o[2 * dp + 1], pa0, pa1, pa2, pa3, b2, b3);
         }

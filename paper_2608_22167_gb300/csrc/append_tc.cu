@@ -39,6 +39,14 @@
 //   o_free[X]          epilogue has read O_X (next item may overwrite it)
 //   q_full/q_empty     query tiles loaded / last QK^T of the item done
 //   item_full/empty[2] two-slot queue of work items from the producer
+//
+// A wait that runs out sets an abort flag in shared memory that every other
+// role's waits poll, so the whole CTA leaves within microseconds; before TMEM
+// is freed the issuers wait for their MMAs and the producer for its copies
+// still in flight. append_tc_kernel<true> is the self-test form of the same
+// kernel (mcpu_selftest_append_abort): one chosen role stops at the second
+// key block of its first item and waits on a barrier nothing completes (for
+// half the wait limit), and each warp reports when it left.
 #include "tcgen05.cuh"
 
 namespace mcpu {
@@ -69,10 +77,12 @@ struct TcSmem {  // barriers and small state, after the tiles
   uint64_t s_full[2], s_free[2], p_full[2], o_ready[2], o_free[2];
   uint64_t item_full[2], item_empty[2];
   uint64_t drain[2];  // each issuer's last MMAs complete (before TMEM is freed)
+  uint64_t never;     // self-test form only: a barrier nothing completes
   AppendItem items[2];
   int32_t item_idx[2];
   uint32_t tmem_base;
-  int32_t abort_flag;
+  int32_t abort_flag;  // 1: a wait ran out; 2: the self-test's stalled role gave up
+  uint64_t t_start;    // self-test form only: %globaltimer at kernel start
 };
 
 size_t append_tc_smem_bytes() {
@@ -157,6 +167,25 @@ __device__ __forceinline__ float chunk_exp(const uint32_t (&sv)[2][32], float sc
   return lo_f32(ls) + hi_f32(ls);
 }
 
+__device__ __forceinline__ void st_shared_zero16(uint32_t addr) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(addr), "r"(0u) : "memory");
+}
+
+// Self-test form only: the stalled role waits on a barrier nothing completes
+// for half the library's wait limit, without polling the abort flag; then it
+// raises the flag with its own mark (2) unless another role already did. The
+// other roles, which began waiting at about the same time with the full
+// limit, must leave on seeing the flag; one that ran out of its own wait
+// instead would overwrite the mark with 1, and leave a half limit later.
+constexpr uint64_t kSelftestStallNs = kWaitTimeoutNs / 2;
+__device__ __forceinline__ void selftest_stall(uint32_t never_bar, int32_t* abort_flag) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait_sleep(never_bar, 0, 10000)) {
+    if (global_timer_ns() - t0 > kSelftestStallNs) break;
+  }
+  atomicCAS(abort_flag, 0, 2);
+}
+
 // Probabilities of one chunk against the running reference m_ref (log2
 // units): p = 2^(s * scale_log2 - m_ref). The common path computes no max:
 // a chunk sum below 2^8 proves every p is below 2^8, the bound the lazy
@@ -185,6 +214,7 @@ __device__ __forceinline__ float chunk_probs(const uint32_t (&sv)[2][32], float 
 
 }  // namespace
 
+template <bool kSelfTest>
 __global__ void __maxnreg__(144)
     append_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap qmap, const AttnParams p) {
@@ -223,7 +253,9 @@ __global__ void __maxnreg__(144)
       mbar_init(bar(st.item_empty[x]), 8 + 2);  // softmax warps and both issuers
       mbar_init(bar(st.drain[x]), 1);
     }
+    mbar_init(bar(st.never), 1);
     st.abort_flag = 0;
+    if (kSelfTest) st.t_start = global_timer_ns();
     fence_barrier_init();
   }
   if (warp == kTcSWarp) {
@@ -252,6 +284,7 @@ __global__ void __maxnreg__(144)
     }
     const uint64_t pol = policy_evict_last();
     uint32_t kv_it = 0;
+    uint32_t k_issued = 0, v_issued = 0, q_issued = 0;  // copies issued so far, per ring
     for (int i = 0;; ++i) {
       const int slot = i & 1;
       if (i >= 2 && !__all_sync(0xffffffffu, wait_bar(bar(st.item_empty[slot]), ((i >> 1) - 1) & 1, abort_flag)))
@@ -291,6 +324,7 @@ __global__ void __maxnreg__(144)
         mbar_arrive_expect_tx(bar(st.q_full), kTcQBytes);
         tma_load_3d(sQ, &qmap, 0, kvh * g, a.token_begin, bar(st.q_full));
       }
+      q_issued = i + 1;
       bool ok = true;
       constexpr int kPagesPerBlock = kTcKeys / kPage;  // 8: four blocks per 32-page chunk
       // K of block b, then V of block b - 1 (same pool rows, kept from the
@@ -311,9 +345,16 @@ __global__ void __maxnreg__(144)
           for (int j = 0; j < kPagesPerBlock; ++j)
             tma_load_2d(dst + j * kTileBytes, is_k ? &kmap : &vmap, 0, y[j], bar(full[s]), pol);
         }
+        (is_k ? k_issued : v_issued) = it + 1;
         return true;
       };
       for (int b = 0; b < nb; ++b, ++kv_it) {
+        if (kSelfTest && p.selftest_stall == 1 && i == 0 && b == 1) {
+          if (lane == 0) selftest_stall(bar(st.never), &st.abort_flag);
+          __syncwarp();
+          ok = false;
+          break;
+        }
         if (b > 0 && (b * kPagesPerBlock) % 32 == 0) {
           pid_cur = pid_next;
           pid_next = load_chunk(b * kPagesPerBlock / 32 + 1);
@@ -334,6 +375,17 @@ __global__ void __maxnreg__(144)
       }
       if (ok && nb > 0 && !load_block(false, kv_it - 1, y_prev)) ok = false;
       if (!ok) break;
+    }
+    // After an abort, copies may still be in flight into the rings: wait
+    // (bounded) for the last ones issued to each ring before the CTA ends.
+    // Each such copy is the latest of its stage, so its full barrier's phase
+    // parity identifies it. A finished kernel has none in flight.
+    if (*abort_flag && lane == 0) {
+      for (uint32_t it = k_issued > (uint32_t)kTcKStages ? k_issued - kTcKStages : 0; it < k_issued; ++it)
+        mbar_wait(bar(st.k_full[it % kTcKStages]), (it / kTcKStages) & 1);
+      for (uint32_t it = v_issued > (uint32_t)kTcVStages ? v_issued - kTcVStages : 0; it < v_issued; ++it)
+        mbar_wait(bar(st.v_full[it % kTcVStages]), (it / kTcVStages) & 1);
+      if (q_issued > 0) mbar_wait(bar(st.q_full), (q_issued - 1) & 1);
     }
   } else if (warp == kTcSWarp || warp == kTcPvWarp) {
     // ---------------------------------------------------------- MMA issuers
@@ -369,6 +421,11 @@ __global__ void __maxnreg__(144)
         const int nb = (a.key_end - kb0 + kTcKeys - 1) / kTcKeys;
         if (!wait_bar(bar(st.q_full), i & 1, abort_flag)) break;
         for (int b = 0; b <= nb && ok; ++b) {
+          if (kSelfTest && p.selftest_stall == 2 && x == 0 && i == 0 && b == 1) {
+            selftest_stall(bar(st.never), &st.abort_flag);
+            ok = false;
+            break;
+          }
           if (b < nb) {  // S_x(b)
             const uint32_t bk = blk + b;
             const int s = bk % kTcKStages;
@@ -445,6 +502,12 @@ __global__ void __maxnreg__(144)
       const int wp_max = a.pos_begin + min(x * tile_tok + (wq * 32 + 31) / g, last_tok);
       float m_ref = -INFINITY, l = 0.f;
       for (int b = 0; b < nb; ++b, ++blk) {
+        if (kSelfTest && p.selftest_stall == 0 && x == 0 && i == 0 && b == 1) {
+          if (lane == 0) selftest_stall(bar(st.never), &st.abort_flag);
+          __syncwarp();
+          ok = false;
+          break;
+        }
         ok = __all_sync(0xffffffffu, wait_bar_poll(bar(st.s_full[x]), blk & 1, abort_flag));
         if (!ok) break;
         tc_fence_after();
@@ -491,6 +554,31 @@ __global__ void __maxnreg__(144)
         }
         tmem_st32(cP + 32, pk);
         l = l * alpha + (l0 + l1);
+        // V rows of slots no query of the item sees (before key_begin on the
+        // partial first page of a window, from key_end on the partial last
+        // page) were perhaps never written and may hold NaN, which a zero
+        // weight does not cancel (0 x NaN = NaN). Once the block's V stage
+        // has landed they are zeroed in shared memory (at most 15 rows each;
+        // whole pages past the row's end arrive as zeros already), then
+        // handed to the async proxy before this tile's PV may read them. Both
+        // tiles' warps write the same zeros, each before its own p_full.
+        {
+          const bool lo_edge = b == 0 && kb0 < a.key_begin;
+          const bool hi_edge = b == nb - 1 && (a.key_end & (kPage - 1)) != 0;
+          if (lo_edge || hi_edge) {
+            const uint32_t sv_i = blk % kTcVStages;
+            ok = __all_sync(0xffffffffu, wait_bar_poll(bar(st.v_full[sv_i]), (blk / kTcVStages) & 1, abort_flag));
+            if (!ok) break;
+            const uint32_t vst = sV + sv_i * kTcKvBytes;
+            const int zr = row >> 3, zc = row & 7;  // key row (0..15) and 16-byte chunk of this thread
+            if (lo_edge && zr < a.key_begin - kb0) st_shared_zero16(vst + zr * kRowBytes + zc * 16);
+            if (hi_edge) {
+              const int r0 = a.key_end - kb;  // first row past the row's end, inside this block
+              if (zr < kPage - (r0 & (kPage - 1))) st_shared_zero16(vst + (r0 + zr) * kRowBytes + zc * 16);
+            }
+            fence_proxy_async();
+          }
+        }
         // O_X may only be rescaled once PV_X(blk - 1) has completed (waited above)
         if (b > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
           uint32_t ov[32];
@@ -548,29 +636,44 @@ __global__ void __maxnreg__(144)
 
   // every role ends here; a timed-out role has set the abort flag
   __syncwarp();
+  if (kSelfTest && lane == 0 && blockIdx.x == 0) p.selftest_report[1 + warp] = (int64_t)(global_timer_ns() - st.t_start);
   if (threadIdx.x == 0 && *abort_flag) raise_status(p, kStatusTimeout);
   tc_fence_before();
   __syncthreads();
   if (warp == kTcSWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
+    if (kSelfTest && lane == 0 && blockIdx.x == 0) {
+      p.selftest_report[0] = *abort_flag;
+      p.selftest_report[12] = (int64_t)kSelftestStallNs;
+      p.selftest_report[13] = (int64_t)kWaitTimeoutNs;
+      p.selftest_report[14] = 1;  // TMEM freed
+    }
   }
 }
 
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                              const AttnParams& p, int grid, cudaStream_t stream) {
-  append_tc_kernel<<<grid, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
+  append_tc_kernel<false><<<grid, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
+  return cudaGetLastError();
+}
+
+// The self-test form: one CTA, p.selftest_stall names the stalled role and
+// p.selftest_report receives the abort flag and each warp's exit time.
+cudaError_t launch_append_tc_selftest(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
+                                      const AttnParams& p, cudaStream_t stream) {
+  append_tc_kernel<true><<<1, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
   return cudaGetLastError();
 }
 
 cudaError_t prepare_append_tc_kernel(int* blocks_per_sm) {
-  cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)append_tc_smem_bytes());
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared);
-  if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_tc_kernel, kTcThreads,
+  for (auto fn : {append_tc_kernel<false>, append_tc_kernel<true>}) {
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_tc_smem_bytes());
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_tc_kernel<false>, kTcThreads,
                                                        append_tc_smem_bytes());
 }
 

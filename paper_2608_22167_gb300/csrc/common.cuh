@@ -128,6 +128,10 @@ struct AttnParams {
   int32_t append_tile_tok;       // tokens per append tile (tile rows / group)
   const float* sinks;            // [Hq] sink logits (natural log), or null
   int32_t decode_only;           // 1: rows with L > 1 are reported and skipped (fp8 pools)
+  // read only by the self-test form of the append kernel: the role that
+  // stalls and the report it writes (mcpu_selftest_append_abort)
+  int32_t selftest_stall = -1;
+  int64_t* selftest_report = nullptr;
 };
 
 // Attention sinks (gpt-oss): q head h has a logit sigma_h that joins the

@@ -203,8 +203,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         for (int i = 0; i < 4; ++i) tv[nt][i] = fmaf(c[nt][i], p.scale_log2, -m_ref[nt][i & 1]);
       // keys outside [first_key, seq_len): only a row's first and last pages
       const int j0 = (pb + k) * kPage + (lane >> 2);
+      const bool edge = NT == 1 && ((pb + k) * kPage < first_key || (pb + k + 1) * kPage > seq_len);
       bool v0 = true, v1 = true;
-      if (NT == 1 && ((pb + k) * kPage < first_key || (pb + k + 1) * kPage > seq_len)) {
+      if (edge) {
         v0 = j0 >= first_key && j0 < seq_len;
         v1 = (j0 + 8) >= first_key && (j0 + 8) < seq_len;
 #pragma unroll
@@ -258,11 +259,29 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         pb1[nt] = movmatrix_trans(pack_bf16x2(p10, p11));
       }
 
+      // V rows of slots outside [first_key, seq_len) were perhaps never
+      // written and may hold NaN, which a zero weight does not cancel
+      // (0 x NaN = NaN): on a row's first and last page they are zeroed in the
+      // operand. This lane's V^T fragments a0/a1 hold keys 2c, 2c + 1 and
+      // a2/a3 keys 2c + 8, 2c + 9 of the page (c = lane & 3), the lower key
+      // in the low half of each word.
+      uint32_t vm_lo = 0xffffffffu, vm_hi = 0xffffffffu;
+      if (edge) {
+        const int jv = (pb + k) * kPage + 2 * (lane & 3);
+        auto seen = [&](int j) { return j >= first_key && j < seq_len; };
+        vm_lo = (seen(jv) ? 0x0000ffffu : 0u) | (seen(jv + 1) ? 0xffff0000u : 0u);
+        vm_hi = (seen(jv + 8) ? 0x0000ffffu : 0u) | (seen(jv + 9) ? 0xffff0000u : 0u);
+      }
+
       // O^T[64 dims x 8*NT] += V^T P^T
 #pragma unroll
       for (int mt = 0; mt < 4; ++mt) {
         uint32_t a0, a1, a2, a3;
         ldmatrix_x4_trans(vt + swz128(ri + (mi >> 1) * 8, 2 * mt + (mi & 1)), a0, a1, a2, a3);
+        a0 &= vm_lo;
+        a1 &= vm_lo;
+        a2 &= vm_hi;
+        a3 &= vm_hi;
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(acc[mt][nt], a0, a1, a2, a3, pb0[nt], pb1[nt]);
       }

@@ -111,6 +111,10 @@ _lib.mcpu_reset_device_status.argtypes = [_P, _P]
 _lib.mcpu_reset_device_status.restype = ctypes.c_int
 _lib.mcpu_selftest_wait_timeout.argtypes = [_P, _P, _P]
 _lib.mcpu_selftest_wait_timeout.restype = ctypes.c_int
+_lib.mcpu_selftest_append_abort.argtypes = [
+    _P, _P, _P, _P, _P, _P, ctypes.c_float, ctypes.POINTER(Dims), _P, _P, _P, ctypes.c_size_t, ctypes.c_int32, _P, _P,
+]
+_lib.mcpu_selftest_append_abort.restype = ctypes.c_int
 _lib.mcpu_status_string.argtypes = [ctypes.c_int]
 _lib.mcpu_status_string.restype = ctypes.c_char_p
 _lib.mcpu_abi_version.argtypes = []
@@ -352,6 +356,26 @@ def mcpu_selftest_wait_timeout(workspace, report, stream=None):
         raise McpuError(1, "mcpu_selftest_wait_timeout")
     _check(_lib.mcpu_selftest_wait_timeout(_ptr(workspace), _ptr(report), _stream(stream)),
            "mcpu_selftest_wait_timeout")
+
+
+def mcpu_selftest_append_abort(q, k_cache, v_cache, block_table, seq_lens, query_start_loc, softmax_scale, out, lse,
+                               workspace, stall_role, report, stream=None):
+    """Enqueues the append kernel's abort self-check as one CTA over this
+    batch: role ``stall_role`` (0 softmax of tile A, 1 producer, 2 issuer of
+    tile A) waits on a barrier nothing completes; ``report`` is a device int64
+    tensor of 16 entries (final abort flag, each warp's exit time in ns, the
+    stalled wait, the wait limit, TMEM freed)."""
+    if report.dtype != torch.int64 or report.numel() < 16 or not report.is_cuda:
+        raise McpuError(1, "mcpu_selftest_append_abort")
+    d = dims(q, k_cache, block_table, seq_lens)
+    _check(
+        _lib.mcpu_selftest_append_abort(
+            _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), _ptr(query_start_loc),
+            float(softmax_scale), ctypes.byref(d), _ptr(out), _ptr(lse), _ptr(workspace),
+            workspace.numel() * workspace.element_size(), int(stall_role), _ptr(report), _stream(stream),
+        ),
+        "mcpu_selftest_append_abort",
+    )
 
 
 def new_workspace(d: Dims, device="cuda") -> torch.Tensor:

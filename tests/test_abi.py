@@ -162,6 +162,26 @@ def test_timeout_selftest_host_checks(lib):
     assert f(P, P + 4, None) == 1  # report not 8-byte aligned
 
 
+def test_append_abort_selftest_host_checks(lib):
+    f = _fn(lib, "mcpu_selftest_append_abort")
+    f.argtypes = [ctypes.c_void_p] * 6 + [ctypes.c_float, ctypes.POINTER(Dims)] + [ctypes.c_void_p] * 3 + \
+        [ctypes.c_size_t, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p]
+    d = Dims(2, 40, 19, 34, 16, 2, 64, 16)
+    lib.mcpu_workspace_size.restype = ctypes.c_size_t
+    need = lib.mcpu_workspace_size(ctypes.byref(d))
+    P = 1 << 20
+    args = lambda role, rep, ws=P, nbytes=need: (P, P, P, P, P, P, 0.125, ctypes.byref(d), P, P, ws,  # noqa: E731
+                                                 nbytes, role, rep, None)
+    assert f(*args(3, P)) == 1  # no such role
+    assert f(*args(-1, P)) == 1
+    assert f(*args(0, None)) == 1  # no report
+    assert f(*args(0, P + 4)) == 1  # report not 8-byte aligned
+    assert f(*args(0, P, ws=P + 16)) == 1  # workspace not 256-byte aligned
+    assert f(*args(0, P, nbytes=need - 1)) == 3  # workspace too small
+    bad = Dims(2, 40, 19, 34, 16, 2, 128, 16)
+    assert f(P, P, P, P, P, P, 0.125, ctypes.byref(bad), P, P, P, need, 0, P, None) == 2  # head_dim 128
+
+
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-GPU error path")
 def test_no_gpu_is_a_clean_error(lib):
     fwd = _fn(lib, "mcpu_paged_attention_forward")

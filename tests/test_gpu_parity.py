@@ -9,9 +9,34 @@ import workloads as W
 
 pytestmark = pytest.mark.gpu
 
+import oracle
+
 if torch.cuda.is_available():
     from _gpu import Run, assert_parity, oracle_full, oracle_sampled
     from paper_2608_22167_gb300 import mcpu
+
+
+def _poison_unseen_slots(batch, layer=0):
+    """Writes NaN into every K and V slot of the layer's pool that no query of
+    the batch can see (slots past a row's end on its last page, slots before
+    a window on its first page, the pool's spare pages), as memory that was
+    never written may hold. The oracle reads visible keys only."""
+    lay = batch.layers[layer]
+    pool = batch.pools[lay.pool]
+    P = pool.k_cache.shape[0]
+    seen = np.zeros((P, 16), bool)
+    bt, S, L = pool.block_table, batch.seq_lens, batch.q_lens
+    W_ = lay.sliding_window
+    for r in range(batch.num_seqs):
+        if L[r] == 0:
+            continue
+        lo = 0 if W_ <= 0 else max(0, int(S[r] - L[r]) - W_ + 1)
+        j = np.arange(lo, int(S[r]))
+        seen[bt[r, j // 16], j % 16] = True
+    hide = torch.from_numpy(~seen)
+    for t in (pool.k_cache, pool.v_cache):
+        t.permute(0, 2, 1, 3)[hide.to(t.device)] = float("nan")
+    return int((~seen).sum())
 
 
 def _full_check(batch, layer=0, flags=0, split_pages=0, what="", sinks=None):
@@ -193,7 +218,70 @@ def test_gqa_ratios(group):
     _full_check(b, what=f"gqa{group}")
 
 
+@pytest.mark.parametrize("case", ["decode", "split", "window", "append", "append_window", "mma_sync", "cascade"])
+def test_unwritten_slots_may_hold_nan(case):
+    # Slots no query can see hold NaN in K and V (never-written memory may):
+    # the kernels mask their scores and zero their V rows, since a zero
+    # weight does not cancel NaN. Every output must match the oracle, which
+    # reads visible keys only.
+    rng = np.random.default_rng(len(case) * 31 + ord(case[0]))
+    flags, split = 0, 0
+    if case == "cascade":
+        b = _grouped_batch(17)
+    else:
+        B = 7
+        S = rng.integers(20, 1500, size=B)
+        S[0] = 16 * 37 + 5  # a partial last page
+        app = case.startswith("append") or case == "mma_sync"
+        L = np.where((np.arange(B) % 2 == 0) & app, np.minimum(S, rng.integers(2, 300, size=B)), 1)
+        win = 100 if case.endswith("window") or case == "window" else 0
+        b = W.build_batch(f"nan_{case}", 500 + len(case), S, L, 64, 8, layer_windows=(win,), pool_slack_pages=5)
+        flags = mcpu.FLAG_MMA_SYNC_APPEND if case == "mma_sync" else 0
+        split = 2 if case == "split" else 0
+    assert _poison_unseen_slots(b) > 0
+    run, _ = _full_check(b, flags=flags, split_pages=split, what=f"NaN in unseen slots ({case})")
+    if case == "cascade":
+        assert run.header()["n_cascade"] > 0
+    if case == "split":
+        assert run.header()["n_merge"] > 0
+
+
 # ---------------------------------------------------------------- full sizes
+
+
+def _appended_pages_bitexact(batch, run, layer=0):
+    """Every page this step's KV append wrote (all rows: one slot per decode
+    row, the whole chunk of an append row), compared bit for bit with the
+    oracle's KV append of those rows: the touched pages are gathered before
+    (from the batch, which the run does not modify) and after the append,
+    into a compact pool with a renumbered block table."""
+    lay = batch.layers[layer]
+    pool = batch.pools[lay.pool]
+    S, L, qsl = batch.seq_lens.astype(np.int64), batch.q_lens.astype(np.int64), batch.query_start_loc
+    rows = np.nonzero(L > 0)[0]
+    bt = pool.block_table
+    touched = np.unique(np.concatenate([bt[r, (S[r] - L[r]) // 16:(S[r] - 1) // 16 + 1] for r in rows]))
+    assert np.all(touched >= 0)
+    remap = np.full(pool.num_pages, -1, np.int64)
+    remap[touched] = np.arange(touched.shape[0])
+    bt_c = np.full((len(rows), bt.shape[1]), -1, np.int32)
+    for i, r in enumerate(rows):
+        lp = np.arange((S[r] - L[r]) // 16, (S[r] - 1) // 16 + 1)
+        bt_c[i, lp] = remap[bt[r, lp]]
+    idx = torch.as_tensor(touched, device=pool.k_cache.device)
+    tok = torch.as_tensor(np.concatenate([np.arange(qsl[r], qsl[r + 1]) for r in rows]), device=lay.k_new.device)
+    qsl_c = np.zeros(len(rows) + 1, np.int32)
+    qsl_c[1:] = np.cumsum(L[rows])
+    want_k, want_v = oracle.kv_append(W.to_host(lay.k_new.index_select(0, tok)),
+                                      W.to_host(lay.v_new.index_select(0, tok)),
+                                      W.to_host(pool.k_cache.index_select(0, idx)),
+                                      W.to_host(pool.v_cache.index_select(0, idx)), bt_c,
+                                      S[rows].astype(np.int32), qsl_c)
+    got_k = W.to_host(run.kc.index_select(0, idx.to(run.kc.device)))
+    got_v = W.to_host(run.vc.index_select(0, idx.to(run.vc.device)))
+    assert np.array_equal(got_k, want_k), f"k pages differ after the append (layer {layer})"
+    assert np.array_equal(got_v, want_v), f"v pages differ after the append (layer {layer})"
+    return int(touched.shape[0])
 
 
 def _sampled_check(batch, rows, n_per_row, seed, layer=0, run=None):
@@ -229,7 +317,12 @@ def test_mixed_batch_sampled():
     dec = list(np.nonzero(L == 1)[0])
     rng = np.random.default_rng(5)
     rows = sorted(app[:6] + list(rng.choice(dec, size=10, replace=False)))
-    _sampled_check(b, rows, n_per_row=24, seed=6)
+    run = Run(b)
+    run.append()
+    run.forward()
+    # the whole step's KV append, every written page bit for bit
+    assert _appended_pages_bitexact(b, run) > 1000
+    _sampled_check(b, rows, n_per_row=24, seed=6, run=run)
 
 
 def test_long_horizon_sampled():
@@ -254,6 +347,7 @@ def test_rollout_step_sampled_every_layer():
         run.forward()
         if b.layers[layer].sliding_window == 0:
             assert run.header()["n_cascade"] > 0
+        _appended_pages_bitexact(b, run, layer)
         _sampled_check(b, rows, n_per_row=6, seed=100 + layer, layer=layer, run=run)
         del run
         torch.cuda.empty_cache()
