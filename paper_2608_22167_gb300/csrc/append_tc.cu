@@ -389,15 +389,19 @@ __global__ void __maxnreg__(144)
     }
   } else if (warp == kTcSWarp || warp == kTcPvWarp) {
     // ---------------------------------------------------------- MMA issuers
-    // One issuing thread per tile (warp 9: tile A, warp 10: tile B), each in
+    // One issuing warp per tile (warp 9: tile A, warp 10: tile B), each in
     // its tile's own order S(b), PV(b - 1), so that neither tile's MMAs wait
-    // behind the other tile's softmax. Their MMAs touch disjoint TMEM and are
+    // behind the other tile's softmax. The whole warp runs the loop in step
+    // and one elected lane issues each MMA: operands computed by a lone lane
+    // of a diverged warp leave the uniform datapath, which costs each MMA
+    // about 50 cycles of issue (a 128 x 64 x 16 MMA computes in 32; the PV
+    // issue of a block went 717 -> 474 cycles). Their MMAs touch disjoint TMEM and are
     // ordered only through the mbarriers; a K or V stage and the query tiles
     // are released by two commits, one per tile. The loops are lean:
     // descriptors are computed once and stepped by constants (the
     // start-address field counts 16-byte units and cannot overflow: shared
     // memory ends below 256 KiB).
-    if (lane == 0) {
+    {
       constexpr uint32_t idS = idesc_bf16(kTcRows, kTcKeys, false, false);
       constexpr uint32_t idO = idesc_bf16(kTcRows, kHeadDim, false, true);
       constexpr uint64_t kStageStep = kTcKvBytes / 16, kVStep = 16 * kRowBytes / 16;
@@ -437,13 +441,13 @@ __global__ void __maxnreg__(144)
             }
             tc_fence_after();
             const uint64_t kd = kdesc0 + s * kStageStep;
-            tc_mma_ss(scol, qd, kd, idS, 0u);
+            tc_mma_ss_e(scol, qd, kd, idS, 0u);
 #pragma unroll
             for (int kk = 1; kk < kHeadDim / 16; ++kk)
-              tc_mma_ss(scol, qd + (uint64_t)(kk * 2), kd + (uint64_t)(kk * 2), idS, 1u);
-            tc_commit(bar(st.s_full[x]));
-            tc_commit(bar(st.k_empty[s]));              // released when both tiles have read it
-            if (b == nb - 1) tc_commit(bar(st.q_empty));  // likewise
+              tc_mma_ss_e(scol, qd + (uint64_t)(kk * 2), kd + (uint64_t)(kk * 2), idS, 1u);
+            tc_commit_e(bar(st.s_full[x]));
+            tc_commit_e(bar(st.k_empty[s]));              // released when both tiles have read it
+            if (b == nb - 1) tc_commit_e(bar(st.q_empty));  // likewise
           }
           if (b >= 1) {  // O_x += P_x(b - 1) V(b - 1)
             const uint32_t bv = blk + b - 1;
@@ -456,20 +460,20 @@ __global__ void __maxnreg__(144)
             }
             tc_fence_after();
             const uint64_t vd = vdesc0 + sv * kStageStep;
-            tc_mma_ts(ocol, pcol, vd, idO, b > 1 ? 1u : 0u);
+            tc_mma_ts_e(ocol, pcol, vd, idO, b > 1 ? 1u : 0u);
 #pragma unroll
-            for (int kk = 1; kk < kTcKeys / 16; ++kk) tc_mma_ts(ocol, pcol + kk * 8, vd + kk * kVStep, idO, 1u);
-            tc_commit(bar(st.o_ready[x]));
-            tc_commit(bar(st.v_empty[sv]));  // released when both tiles have read it
+            for (int kk = 1; kk < kTcKeys / 16; ++kk) tc_mma_ts_e(ocol, pcol + kk * 8, vd + kk * kVStep, idO, 1u);
+            tc_commit_e(bar(st.o_ready[x]));
+            tc_commit_e(bar(st.v_empty[sv]));  // released when both tiles have read it
           }
         }
         if (!ok) break;
         blk += nb;
-        mbar_arrive(bar(st.item_empty[slot]));
+        if (lane == 0) mbar_arrive(bar(st.item_empty[slot]));
       }
       // wait for this thread's MMAs still in flight (only after an abort can
       // any be), so that TMEM is not freed under them
-      tc_commit(bar(st.drain[x]));
+      tc_commit_e(bar(st.drain[x]));
       mbar_wait(bar(st.drain[x]), 0);
     }
   } else {
