@@ -656,57 +656,60 @@ def run_ours(args, rank, world, dev):
     # copies q / k_new / v_new in and out / lse back, overlapped with the
     # compute by row slices; the step ends when its last output is in host
     # memory.
-    lay_host = []
-    for lay in batch.layers:
-        lay_host.append((lay.q.cpu().pin_memory(), lay.k_new.cpu().pin_memory(), lay.v_new.cpu().pin_memory()))
-    meta_host = [torch.from_numpy(batch.seq_lens).to(torch.int32).pin_memory(),
-                 torch.from_numpy(batch.query_start_loc).to(torch.int32).pin_memory()]
-    bt_host = {k: torch.from_numpy(p.block_table).pin_memory() for k, p in batch.pools.items()}
-    q0 = batch.layers[0].q
-    out_h = torch.empty(q0.shape, dtype=q0.dtype).pin_memory()
-    lse_h = torch.empty(q0.shape[:2], dtype=torch.float32).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for tr in lay_host for t in tr)
-    h2d += sum(t.numel() * t.element_size() for t in meta_host) + sum(
-        t.numel() * t.element_size() for t in bt_host.values())
-    d2h = (out_h.numel() * out_h.element_size() + lse_h.numel() * 4) * nl
-    host_stage = mcpu.HostStage(q0.shape[0], batch.num_seqs, batch.num_q_heads, batch.num_kv_heads, slots=3)
+    e2e_steps = 0 if getattr(args, "skip_e2e", False) else max(3, min(args.steps, 20))
+    h2d = d2h = 0
+    e2e_ms = e2e_median_ms = float("nan")
+    if e2e_steps:
+        lay_host = []
+        for lay in batch.layers:
+            lay_host.append((lay.q.cpu().pin_memory(), lay.k_new.cpu().pin_memory(), lay.v_new.cpu().pin_memory()))
+        meta_host = [torch.from_numpy(batch.seq_lens).to(torch.int32).pin_memory(),
+                     torch.from_numpy(batch.query_start_loc).to(torch.int32).pin_memory()]
+        bt_host = {k: torch.from_numpy(p.block_table).pin_memory() for k, p in batch.pools.items()}
+        q0 = batch.layers[0].q
+        out_h = torch.empty(q0.shape, dtype=q0.dtype).pin_memory()
+        lse_h = torch.empty(q0.shape[:2], dtype=torch.float32).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for tr in lay_host for t in tr)
+        h2d += sum(t.numel() * t.element_size() for t in meta_host) + sum(
+            t.numel() * t.element_size() for t in bt_host.values())
+        d2h = (out_h.numel() * out_h.element_size() + lse_h.numel() * 4) * nl
+        host_stage = mcpu.HostStage(q0.shape[0], batch.num_seqs, batch.num_q_heads, batch.num_kv_heads, slots=3)
 
-    def e2e_step():
-        for key, t in bt_host.items():
-            st.bts[key].copy_(t, non_blocking=True)
-        for i in range(nl):
-            lay = batch.layers[i]
-            qh, knh, vnh = lay_host[i]
-            if fp8:
-                mcpu.mcpu_paged_attention_host_fp8(host_stage, qh, knh, vnh, st.pools8[lay.pool], st.bts[lay.pool],
-                                                   meta_host[0], meta_host[1], lay.sliding_window,
+        def e2e_step():
+            for key, t in bt_host.items():
+                st.bts[key].copy_(t, non_blocking=True)
+            for i in range(nl):
+                lay = batch.layers[i]
+                qh, knh, vnh = lay_host[i]
+                if fp8:
+                    mcpu.mcpu_paged_attention_host_fp8(host_stage, qh, knh, vnh, st.pools8[lay.pool], st.bts[lay.pool],
+                                                       meta_host[0], meta_host[1], lay.sliding_window,
+                                                       batch.softmax_scale, out_h, lse_h, st.ws)
+                else:
+                    pool = batch.pools[lay.pool]
+                    mcpu.mcpu_paged_attention_host(host_stage, qh, knh, vnh, pool.k_cache, pool.v_cache,
+                                                   st.bts[lay.pool], meta_host[0], meta_host[1], lay.sliding_window,
                                                    batch.softmax_scale, out_h, lse_h, st.ws)
-            else:
-                pool = batch.pools[lay.pool]
-                mcpu.mcpu_paged_attention_host(host_stage, qh, knh, vnh, pool.k_cache, pool.v_cache,
-                                               st.bts[lay.pool], meta_host[0], meta_host[1], lay.sliding_window,
-                                               batch.softmax_scale, out_h, lse_h, st.ws)
-        mcpu.mcpu_host_stage_wait(host_stage)
+            mcpu.mcpu_host_stage_wait(host_stage)
 
-    e2e_steps = max(3, min(args.steps, 20))
-    for _ in range(2):
-        e2e_step()
-    torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
-    ev[0].record(stream)
-    for k in range(e2e_steps):
-        e2e_step()
-        ev[k + 1].record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = ev[0].elapsed_time(ev[-1]) / e2e_steps
-    # per-step spread: host-to-device copies out of a multi-GB page-locked
-    # working set can stall for a pass (plain copies do too); the median
-    # shows a typical step, the mean (the reported value) includes stalls
-    e2e_median_ms = statistics.median(ev[k].elapsed_time(ev[k + 1]) for k in range(e2e_steps))
-    mcpu.mcpu_host_stage_sync(host_stage)
-    host_stage.close()
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
+        ev[0].record(stream)
+        for k in range(e2e_steps):
+            e2e_step()
+            ev[k + 1].record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = ev[0].elapsed_time(ev[-1]) / e2e_steps
+        # per-step spread: host-to-device copies out of a multi-GB page-locked
+        # working set can stall for a pass (plain copies do too); the median
+        # shows a typical step, the mean (the reported value) includes stalls
+        e2e_median_ms = statistics.median(ev[k].elapsed_time(ev[k + 1]) for k in range(e2e_steps))
+        mcpu.mcpu_host_stage_sync(host_stage)
+        host_stage.close()
 
     # ---- max over ranks
     total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], dev, world)
@@ -762,7 +765,7 @@ def run_ours(args, rank, world, dev):
         "roofline_decode": roof_dec,
         "roofline_append": roof_app,
         "gpu_launches": st.launches_per_step * args.steps,
-        "e2e": {"value": round(e2e_value, 2), "unit": "GB/s", "h2d_bytes_per_step": int(h2d),
+        "e2e": None if not e2e_steps else {"value": round(e2e_value, 2), "unit": "GB/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "ms_per_step": round(e2e_ms, 4),
                 "median_step_ms": round(e2e_median_ms, 4),
                 "call": ("mcpu_paged_attention_host_fp8" if fp8 else "mcpu_paged_attention_host") +
@@ -907,6 +910,34 @@ def run_churn(args, rank, world, dev):
     }
 
 
+# The other four configurations, each timed the same way as the headline (CUDA
+# graphs of whole steps, events on the launching stream, clocks sampled) but
+# for a fixed, short number of steps, so that one default run measures all
+# five: (workload, timed steps). No CPU baseline and no end-to-end leg here.
+OTHER_CONFIGS = (("tiny", 200), ("decode", 100), ("long", 20), ("rollout", 8))
+
+
+def other_configs(args, rank, world, dev):
+    out = {}
+    for name, steps in OTHER_CONFIGS:
+        sub = argparse.Namespace(**vars(args))
+        sub.workload, sub.steps, sub.warmup = name, steps, 3
+        sub.no_cpu_baseline, sub.compare_launch, sub.skip_e2e = True, False, True
+        r = run_ours(sub, rank, world, dev)
+        rf = r["roofline"] or {}
+        out[name] = {"workload": r["config"]["workload"], "value": r["value"], "unit": r["unit"],
+                     "ms_per_step": r["ms_per_step"], "steps": steps,
+                     "attended_tokens_per_s": r["attended_tokens_per_s"],
+                     "frac_of_hbm_peak": r["frac_of_hbm_peak"], "combined_roofline": r["combined_roofline"],
+                     "roofline": {k: rf.get(k) for k in ("bound", "kernel", "achieved", "peak", "unit", "frac",
+                                                         "traffic", "ms_per_step")},
+                     "kernel_ms_per_step": r["kernel_ms_per_step"], "gpu_launches": r["gpu_launches"],
+                     "clocks": r["clocks"]}
+        del r
+        torch.cuda.empty_cache()
+    return out
+
+
 def run_reference(args, rank, world):
     """The oracle (plain CPU definition) timed on the host cores, rank 0 only."""
     if rank != 0:
@@ -966,6 +997,9 @@ def main():
                     help="time CUDA-graph replays of the whole step (default) or eager C-ABI calls")
     ap.add_argument("--no-compare-launch", dest="compare_launch", action="store_false",
                     help="skip timing the other launch mode")
+    ap.add_argument("--no-other-configs", dest="other_configs", action="store_false",
+                    help="with the default workload on one GPU: skip the short runs of the other four "
+                         "configurations that are added to the line under 'configs'")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -988,6 +1022,9 @@ def main():
 
         build()
         res = run_churn(args, rank, world, dev) if args.workload == "churn" else run_ours(args, rank, world, dev)
+        if (world == 1 and args.workload == "mixed" and args.kv == "bf16" and args.other_configs
+                and args.launch == "graph"):
+            res["configs"] = other_configs(args, rank, world, dev)
     if rank == 0 and res is not None:
         print(json.dumps(res))
     if world > 1:

@@ -413,10 +413,18 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
     it.pad = 0;
     ditems[e] = it;
   }
+  // Cascade records of one group go split-major: (split k, subgroup s) at
+  // the group's base + k * nsub + s, so the subgroups of a group (g = 8:
+  // two of 4 rows) read the same pages within a few tickets of each other
+  // and the second read of each page is an L2 hit, not a second HBM read.
   for (int e = tid; e < tot_cascade; e += NT) {
     const int r = owner_row(sm.sg_off, B, e);
     const int k = e - sm.sg_off[r];
-    const int gp = sm.grp_pages[sm.gid[r]];
+    const int g = sm.gid[r];
+    const int gp = sm.grp_pages[g];
+    const int nd = sm.grp_ndec[g], nsub = cdiv(nd, sub_cap);
+    const int s = (sm.mrank[r] - sm.grp_base[g]) * nsub / nd;
+    const int dst = sm.sg_off[r] - s * sm.n_cs[r] + k * nsub + s;
     CascadeItem c;
     c.member_off = sm.sub_first_idx[r];
     c.n_members = sm.sub_n[r];
@@ -425,7 +433,7 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
     c.split = k;
     c.first_row = r;
     c.pad0 = c.pad1 = 0;
-    citems[e] = c;
+    citems[dst] = c;
   }
   for (int e = tid; e < tot_tiles; e += NT) {
     const int i = owner_row(sm.app_off, n_app, e);
