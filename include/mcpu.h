@@ -101,6 +101,7 @@ typedef struct mcpu_dims {
 #define MCPU_FLAG_NO_CASCADE 0x1u       /* never run the shared-prefix (cascade) pass */
 #define MCPU_FLAG_MMA_SYNC_APPEND 0x2u  /* append chunks on the mma.sync kernel instead of tcgen05 */
 #define MCPU_FLAG_SERIAL 0x4u           /* run every kernel on `stream` (no side stream) */
+#define MCPU_FLAG_HOST_OUT_DIRECT 0x8u  /* host-buffer calls: kernels write out/lse straight into page-locked host memory */
 typedef struct mcpu_options {
   uint32_t flags;             /* MCPU_FLAG_* */
   int32_t split_pages;        /* > 0: KV split length of decode rows, in pages (0 = auto) */
@@ -328,7 +329,15 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
  * slices from 64 MiB moved, else one; a single row is never cut). Slice s's inputs are copied in on the
  * stage's input stream while slice s - 1 computes, and its outputs are
  * copied out on the output stream while slice s + 1 computes; the compute
- * runs on `stream`, ordered after the work already there. Shared-prefix
+ * runs on `stream`, ordered after the work already there.
+ * With MCPU_FLAG_HOST_OUT_DIRECT in opts, and out_host and lse_host in
+ * page-locked memory the device can address, the kernels write the outputs
+ * there themselves as they finish them, over the host link, and nothing is
+ * copied back (slices = 0 then means one slice). That suits the call whose
+ * outputs are wanted right after it (nothing is left to copy once its last
+ * kernel ends); a call followed by more work does better with the copies,
+ * which run beside that work. Without the flag, or for other host memory,
+ * the outputs are staged and copied. Shared-prefix
  * detection only sees rows within one slice. query_start_loc_host is read
  * on the host during the call; the other host buffers are read or written
  * asynchronously: page-locked memory gives full copy speed, and every host

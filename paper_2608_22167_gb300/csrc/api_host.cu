@@ -8,6 +8,10 @@
 // The copy engines of a GB300 move about 210 GB/s host to device and
 // 190 GB/s back, both at once, so a layer whose copies take less than its
 // compute hides them except for the first slice in and the last slice out.
+// With MCPU_FLAG_HOST_OUT_DIRECT and page-locked outputs the kernels write
+// out and lse over the host link themselves (SM stores reach the same
+// ~190 GB/s as the copy engine), so nothing is left to move after the
+// call's last kernel.
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -212,7 +216,7 @@ mcpu_status host_call(mcpu_host_stage* hs, const void* q_host, const void* k_new
                       const int32_t* block_table, const int32_t* seq_lens_host,
                       const int32_t* query_start_loc_host, float softmax_scale, const mcpu_dims* dims,
                       void* out_host, float* lse_host, void* workspace, size_t workspace_bytes, int32_t slices,
-                      mcpu_stream_t stream, Compute compute) {
+                      bool out_direct_wanted, mcpu_stream_t stream, Compute compute) {
   if (!hs || !dims || !seq_lens_host || !query_start_loc_host) return MCPU_ERR_INVALID_ARG;
   if (!on_stage_device(hs)) return MCPU_ERR_INVALID_ARG;
   const int32_t B = dims->num_seqs, T = dims->total_q;
@@ -232,9 +236,27 @@ mcpu_status host_call(mcpu_host_stage* hs, const void* q_host, const void* k_new
   if (T == 0 || B == 0) return MCPU_OK;
   if (!q_host || !k_new_host || !v_new_host || !out_host || !lse_host || !block_table) return MCPU_ERR_INVALID_ARG;
 
+  // outputs written by the kernels themselves: page-locked host memory the
+  // device can address, and the caller asked for it
+  uint8_t* out_direct = nullptr;
+  uint8_t* lse_direct = nullptr;
+  if (out_direct_wanted) {
+    cudaPointerAttributes ao, al;
+    if (cudaPointerGetAttributes(&ao, out_host) == cudaSuccess && ao.type == cudaMemoryTypeHost &&
+        ao.devicePointer != nullptr && cudaPointerGetAttributes(&al, lse_host) == cudaSuccess &&
+        al.type == cudaMemoryTypeHost && al.devicePointer != nullptr) {
+      out_direct = static_cast<uint8_t*>(ao.devicePointer);
+      lse_direct = static_cast<uint8_t*>(al.devicePointer);
+    }
+    (void)cudaGetLastError();  // a query of memory CUDA does not know is not an error of this call
+  }
+
   const int64_t q_row = (int64_t)dims->num_q_heads * kRowBytes, kv_row = (int64_t)dims->num_kv_heads * kRowBytes;
   const int64_t lse_row = (int64_t)dims->num_q_heads * 4;
-  if (slices == 0) slices = (int64_t)T * (2 * q_row + 2 * kv_row + lse_row) >= kTwoSliceBytes ? 2 : 1;
+  // automatic slices: split only to hide copies back (the inputs of a call
+  // are copied while the previous one computes)
+  if (slices == 0)
+    slices = (!out_direct && (int64_t)T * (2 * q_row + 2 * kv_row + lse_row) >= kTwoSliceBytes) ? 2 : 1;
   int32_t rb[MCPU_MAX_HOST_SLICES + 1];
   const int32_t n = mcpu_host_slice_rows(query_start_loc_host, B, slices, rb);
 
@@ -285,10 +307,11 @@ mcpu_status host_call(mcpu_host_stage* hs, const void* q_host, const void* k_new
     c.q = sl.q + t0 * q_row;
     c.k_new = sl.kn + t0 * kv_row;
     c.v_new = sl.vn + t0 * kv_row;
-    c.out = sl.out + t0 * q_row;
-    c.lse = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sl.lse) + t0 * lse_row);
+    c.out = (out_direct ? out_direct : sl.out) + t0 * q_row;
+    c.lse = reinterpret_cast<float*>((lse_direct ? lse_direct : reinterpret_cast<uint8_t*>(sl.lse)) + t0 * lse_row);
     const mcpu_status st = compute(c);
     if (st != MCPU_OK) return fail_after_enqueue(hs, sl, s, st);
+    if (out_direct) continue;  // written in place by the kernels
     // its outputs, once computed
     e = cudaEventRecord(hs->ev_done[k], s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(hs->out, hs->ev_done[k], 0);
@@ -299,7 +322,11 @@ mcpu_status host_call(mcpu_host_stage* hs, const void* q_host, const void* k_new
                           cudaMemcpyDeviceToHost, hs->out);
     if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
   }
-  e = cudaEventRecord(sl.free, hs->out);
+  if (out_direct) {  // the output stream follows the compute, as after copies
+    e = cudaEventRecord(hs->ev_done[0], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(hs->out, hs->ev_done[0], 0);
+  }
+  if (e == cudaSuccess) e = cudaEventRecord(sl.free, hs->out);
   if (e == cudaSuccess) e = cudaEventRecord(hs->ev_out, hs->out);
   if (e != cudaSuccess) return fail_after_enqueue(hs, sl, s, MCPU_ERR_CUDA);
   hs->any_out = true;
@@ -320,7 +347,8 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
   if (!k_cache || !v_cache) return MCPU_ERR_INVALID_ARG;
   int32_t* status = static_cast<int32_t*>(workspace);
   return host_call(hs, q_host, k_new_host, v_new_host, block_table, seq_lens_host, query_start_loc_host,
-                   softmax_scale, dims, out_host, lse_host, workspace, workspace_bytes, slices, stream,
+                   softmax_scale, dims, out_host, lse_host, workspace, workspace_bytes, slices,
+                   opts && (opts->flags & MCPU_FLAG_HOST_OUT_DIRECT), stream,
                    [&](const Slice& c) {
                      mcpu_status st = mcpu_kv_append(c.k_new, c.v_new, k_cache, v_cache, c.block_table, c.seq_lens,
                                                      c.query_start_loc, &c.dims, status, stream);
@@ -340,7 +368,8 @@ mcpu_status mcpu_paged_attention_host_fp8(mcpu_host_stage* hs, const void* q_hos
   if (!kv8) return MCPU_ERR_INVALID_ARG;
   int32_t* status = static_cast<int32_t*>(workspace);
   return host_call(hs, q_host, k_new_host, v_new_host, block_table, seq_lens_host, query_start_loc_host,
-                   softmax_scale, dims, out_host, lse_host, workspace, workspace_bytes, slices, stream,
+                   softmax_scale, dims, out_host, lse_host, workspace, workspace_bytes, slices,
+                   opts && (opts->flags & MCPU_FLAG_HOST_OUT_DIRECT), stream,
                    [&](const Slice& c) {
                      mcpu_status st = mcpu_kv_append_fp8(c.k_new, c.v_new, kv8, c.block_table, c.seq_lens,
                                                          c.query_start_loc, &c.dims, status, stream);

@@ -39,6 +39,7 @@ STATUS = {
 FLAG_NO_CASCADE = 0x1
 FLAG_MMA_SYNC_APPEND = 0x2
 FLAG_SERIAL = 0x4
+FLAG_HOST_OUT_DIRECT = 0x8
 
 # Device status bits (first word of the workspace).
 STATUS_BAD_PAGE = 1

@@ -98,6 +98,32 @@ def test_host_call_pageable_buffers():
     st.close()
 
 
+@pytest.mark.parametrize("pinned", [True, False])
+def test_direct_outputs_equal_the_staged_ones_bitwise(pinned):
+    # MCPU_FLAG_HOST_OUT_DIRECT: the kernels write out / lse straight into
+    # page-locked host memory (ordinary host memory falls back to the copies);
+    # the same kernels run either way, so the results are identical
+    b = W.fuzz_batch(3300 + int(pinned), max_len=1500, max_chunk=300)
+    hc = HostCall(b, pinned=pinned)
+    st = hc.stage()
+    hc.call(st, slices=2)
+    mcpu.mcpu_host_stage_sync(st)
+    hc.check("staged outputs")
+    ref_out, ref_lse = hc.out.clone(), hc.lse.clone()
+    hc.out.fill_(float("nan"))
+    hc.lse.fill_(float("nan"))
+    hc.kc.copy_(b.pools[b.layers[0].pool].k_cache.to("cuda"))
+    hc.vc.copy_(b.pools[b.layers[0].pool].v_cache.to("cuda"))
+    mcpu.mcpu_reset_device_status(hc.ws)
+    mcpu.mcpu_paged_attention_host(st, hc.q, hc.k_new, hc.v_new, hc.kc, hc.vc, hc.bt, hc.sl, hc.qsl, hc.window,
+                                   b.softmax_scale, hc.out, hc.lse, hc.ws, flags=mcpu.FLAG_HOST_OUT_DIRECT)
+    mcpu.mcpu_host_stage_sync(st)
+    hc.check("direct outputs")
+    assert torch.equal(hc.out.view(torch.int16), ref_out.view(torch.int16))
+    assert torch.equal(hc.lse, ref_lse)
+    st.close()
+
+
 def test_one_slice_equals_the_device_call_bitwise():
     b = W.build_batch("host_vs_dev", 3200, np.array([900, 40, 2500, 16, 700]), np.array([1, 17, 300, 1, 1]), 64, 8)
     hc = HostCall(b)
