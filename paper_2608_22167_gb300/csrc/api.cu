@@ -172,7 +172,7 @@ mcpu_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MCPU_OK : cuda_
 
 extern "C" {
 
-int32_t mcpu_abi_version(void) { return 6; }
+int32_t mcpu_abi_version(void) { return 7; }
 
 int32_t mcpu_last_cuda_error(void) { return mcpu::t_last_cuda_error; }
 
