@@ -6,12 +6,21 @@
 //   b = b_max + log2(sum_i 2^(b_i - b_max)),  out = sum_i 2^(b_i - b) o_i,
 // and the reported lse is b * ln 2. An attention sink sigma adds a part
 // 2^(sigma log2 e) with no value. One warp merges one (row, head); each
-// lane owns two of the 64 dims.
+// lane owns two of the 64 dims. The parts' loads are issued together (their
+// normalisers one per lane, their outputs four at a time), so a row costs a
+// few memory round trips, not two per part; the sums still run in part
+// order.
 #include "common.cuh"
 
 namespace mcpu {
 
 constexpr int kMergeWarps = 8;
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
 
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParams p) {
   const PlanHeader* hdr = header(p);
@@ -24,20 +33,44 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
   for (int w = blockIdx.x * kMergeWarps + (threadIdx.x >> 5); w < n; w += gridDim.x * kMergeWarps) {
     const MergeRow mr = rows[w / Hq];
     const int h = w % Hq;
-    float bmax = -INFINITY;
-    for (int i = 0; i < mr.n_parts; ++i) bmax = fmaxf(bmax, lse_part[(size_t)(mr.part_off + i) * Hq + h]);
     // an attention sink joins the normaliser as one more part with no value
     const float s2 = sink_log2(p, h);
-    bmax = fmaxf(bmax, s2);
+    // the parts' log normalisers, 32 at a time (lane i holds part base + i),
+    // so that their loads are in flight together
+    float bmax = s2;
+    for (int base = 0; base < mr.n_parts; base += 32) {
+      const int i = base + lane;
+      const float b = i < mr.n_parts ? lse_part[(size_t)(mr.part_off + i) * Hq + h] : -INFINITY;
+      bmax = fmaxf(bmax, warp_max(b));
+    }
     float sum = s2 > -INFINITY ? fast_exp2(s2 - bmax) : 0.f, o0 = 0.f, o1 = 0.f;
     if (bmax != -INFINITY) {
-      for (int i = 0; i < mr.n_parts; ++i) {
-        const size_t idx = (size_t)(mr.part_off + i) * Hq + h;
-        const float wgt = fast_exp2(lse_part[idx] - bmax);
-        const float2 v = reinterpret_cast<const float2*>(o_part + idx * kHeadDim)[lane];
-        sum += wgt;
-        o0 += wgt * v.x;
-        o1 += wgt * v.y;
+      for (int base = 0; base < mr.n_parts; base += 32) {
+        const int i = base + lane, cnt = min(32, mr.n_parts - base);
+        const float wl = i < mr.n_parts ? fast_exp2(lse_part[(size_t)(mr.part_off + i) * Hq + h] - bmax) : 0.f;
+        const float2* vp = reinterpret_cast<const float2*>(o_part + ((size_t)(mr.part_off + base) * Hq + h) * kHeadDim);
+        const size_t vstride = (size_t)Hq * kHeadDim / 2;  // float2 elements from one part to the next
+        // parts in order (the same sums as one part at a time), four loads in flight
+        int j = 0;
+        for (; j + 4 <= cnt; j += 4) {
+          float2 v[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) v[u] = vp[(j + u) * vstride + lane];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float wgt = __shfl_sync(0xffffffffu, wl, j + u);
+            sum += wgt;
+            o0 += wgt * v[u].x;
+            o1 += wgt * v[u].y;
+          }
+        }
+        for (; j < cnt; ++j) {
+          const float2 v = vp[j * vstride + lane];
+          const float wgt = __shfl_sync(0xffffffffu, wl, j);
+          sum += wgt;
+          o0 += wgt * v.x;
+          o1 += wgt * v.y;
+        }
       }
     }
     const float inv = sum > 0.f ? 1.f / sum : 0.f;
