@@ -666,6 +666,15 @@ def run_ours(args, rank, world, dev):
         meta_host = [torch.from_numpy(batch.seq_lens).to(torch.int32).pin_memory(),
                      torch.from_numpy(batch.query_start_loc).to(torch.int32).pin_memory()]
         bt_host = {k: torch.from_numpy(p.block_table).pin_memory() for k, p in batch.pools.items()}
+        # each step's block tables go into one of two device copies on a copy
+        # stream of their own, so the copy overlaps the previous step instead
+        # of queueing on the compute stream behind it (and behind the stage's
+        # input copies on the same engine)
+        bt_dev = [{k: v.clone() for k, v in st.bts.items()} for _ in range(2)]
+        bt_stream = torch.cuda.Stream()
+        bt_ready = [torch.cuda.Event(), torch.cuda.Event()]
+        bt_free = [torch.cuda.Event(), torch.cuda.Event()]
+        e2e_count = [0]
         q0 = batch.layers[0].q
         out_h = torch.empty(q0.shape, dtype=q0.dtype).pin_memory()
         lse_h = torch.empty(q0.shape[:2], dtype=torch.float32).pin_memory()
@@ -676,8 +685,15 @@ def run_ours(args, rank, world, dev):
         host_stage = mcpu.HostStage(q0.shape[0], batch.num_seqs, batch.num_q_heads, batch.num_kv_heads, slots=3)
 
         def e2e_step():
-            for key, t in bt_host.items():
-                st.bts[key].copy_(t, non_blocking=True)
+            j = e2e_count[0] % 2
+            e2e_count[0] += 1
+            bts = bt_dev[j]
+            with torch.cuda.stream(bt_stream):
+                bt_stream.wait_event(bt_free[j])  # the step two back is done with this copy
+                for key, t in bt_host.items():
+                    bts[key].copy_(t, non_blocking=True)
+                bt_ready[j].record(bt_stream)
+            stream.wait_event(bt_ready[j])
             for i in range(nl):
                 lay = batch.layers[i]
                 qh, knh, vnh = lay_host[i]
@@ -686,15 +702,16 @@ def run_ours(args, rank, world, dev):
                 # it); earlier layers' copies back run beside the next layers
                 fl = mcpu.FLAG_HOST_OUT_DIRECT if i == nl - 1 else 0
                 if fp8:
-                    mcpu.mcpu_paged_attention_host_fp8(host_stage, qh, knh, vnh, st.pools8[lay.pool], st.bts[lay.pool],
+                    mcpu.mcpu_paged_attention_host_fp8(host_stage, qh, knh, vnh, st.pools8[lay.pool], bts[lay.pool],
                                                        meta_host[0], meta_host[1], lay.sliding_window,
                                                        batch.softmax_scale, out_h, lse_h, st.ws, flags=fl)
                 else:
                     pool = batch.pools[lay.pool]
                     mcpu.mcpu_paged_attention_host(host_stage, qh, knh, vnh, pool.k_cache, pool.v_cache,
-                                                   st.bts[lay.pool], meta_host[0], meta_host[1], lay.sliding_window,
+                                                   bts[lay.pool], meta_host[0], meta_host[1], lay.sliding_window,
                                                    batch.softmax_scale, out_h, lse_h, st.ws, flags=fl)
             mcpu.mcpu_host_stage_wait(host_stage)
+            bt_free[j].record(stream)
 
         for _ in range(2):
             e2e_step()
