@@ -53,3 +53,12 @@ def test_whole_job_value_counts_every_rank():
     assert bench.whole_job_gbs(10**9, 1, 1000.0) == pytest.approx(1.0)
     assert bench.whole_job_gbs(10**9, 4, 1000.0) == pytest.approx(4.0)
     assert bench.max_over_ranks([3.0, 4.0], "cpu", 1) == [3.0, 4.0]
+
+
+def test_default_run_covers_every_configuration():
+    # one default bench run times the mixed headline and, under "configs",
+    # the other four configurations of the workload recipe
+    names = {n for n, _ in bench.OTHER_CONFIGS}
+    assert names | {"mixed"} == {"tiny", "decode", "mixed", "long", "rollout"}
+    assert names <= set(W.CONFIGS)
+    assert all(steps >= 8 for _, steps in bench.OTHER_CONFIGS)
