@@ -12,10 +12,10 @@
 #include "common.cuh"
 
 namespace mcpu {
-cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream);
+cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream, bool programmatic);
 cudaError_t prepare_plan_kernel();
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
-                          bool cascade, cudaStream_t stream);
+                          bool cascade, cudaStream_t stream, bool programmatic);
 cudaError_t prepare_decode_kernels(int* bpsm_decode, int* bpsm_cascade);
 cudaError_t launch_append(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
                           cudaStream_t stream);
@@ -25,7 +25,7 @@ cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, c
 cudaError_t launch_append_tc_selftest(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                                       const AttnParams& p, cudaStream_t stream);
 cudaError_t prepare_append_tc_kernel(int* bpsm);
-cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream, bool programmatic);
 cudaError_t prepare_merge_kernel();
 cudaError_t prepare_kv_append_kernel();
 cudaError_t launch_rope_append(void* q, const void* k_new, const void* v_new, void* k_cache, void* v_cache,
@@ -44,7 +44,8 @@ cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* kv8
                                  const int32_t* seq_lens, const int32_t* qsl, int32_t* status, int32_t num_seqs,
                                  int32_t total_q, int32_t max_pages, int32_t num_pages, int32_t num_kv_heads,
                                  cudaStream_t stream);
-cudaError_t launch_decode_fp8(const void* kv8, const AttnParams& p, int grid, bool cascade, cudaStream_t stream);
+cudaError_t launch_decode_fp8(const void* kv8, const AttnParams& p, int grid, bool cascade, cudaStream_t stream,
+                              bool programmatic);
 cudaError_t prepare_fp8_kernels(int* bpsm_decode, int* bpsm_cascade);
 }  // namespace mcpu
 
@@ -328,44 +329,52 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   };
   const bool serial = opts && (opts->flags & MCPU_FLAG_SERIAL);
   const bool cascade = p.cascade_enabled && p.window == 0;
+  // Programmatic launches (the planner after the prefix scan, the cascade
+  // pass after the decode kernel, the merge after the cascade pass) overlap
+  // a launch with the grid before it; not when phase events are recorded
+  // between the kernels.
+  const bool pdl = ev == nullptr;
+  auto merge_grid = [&]() {
+    const int want = (p.num_seqs * p.num_q_heads + 7) / 8;
+    return want < dev->sms * 8 ? (want > 0 ? want : 1) : dev->sms * 8;
+  };
   auto launch_append_kernel = [&]() -> cudaError_t {
     if (legacy_append) return launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
     return launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
   };
   cudaError_t e = mark(0, s);
-  if (e == cudaSuccess) e = launch_plan(p, s);
+  if (e == cudaSuccess) e = launch_plan(p, s, pdl);
   if (e == cudaSuccess) e = mark(1, s);
   if (serial) {
-    if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s);
+    if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s, false);
     if (e == cudaSuccess) e = mark(2, s);
-    if (e == cudaSuccess && cascade) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, s);
+    if (e == cudaSuccess && cascade) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, s, pdl);
     if (e == cudaSuccess) e = mark(3, s);
     if (e == cudaSuccess) e = launch_append_kernel();
     if (e == cudaSuccess) e = mark(4, s);
+    if (e == cudaSuccess) e = launch_merge(p, merge_grid(), s, false);
   } else {
     // fork: the append kernel goes first on `stream` (its CTAs claim the
     // SMs); the decode kernel follows on the low-priority side stream and its
     // CTAs (few registers) fill the room each SM has left. The cascade pass
     // comes after decode on the side stream: its CTAs need more registers
     // than an SM running an append CTA has free, so it may only start as the
-    // append kernel drains. Join before the merge.
+    // append kernel drains. The merge, which reads only decode and cascade
+    // partials and writes only split decode rows, ends the side stream's
+    // chain, so it can run while the append kernel still does. Join last.
     std::lock_guard<std::mutex> lock(dev->fork_mu);
     if (e == cudaSuccess) e = cudaEventRecord(dev->ev_fork, s);
     if (e == cudaSuccess) e = launch_append_kernel();
     if (e == cudaSuccess) e = mark(4, s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(dev->side, dev->ev_fork, 0);
-    if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, dev->side);
+    if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, dev->side, false);
     if (e == cudaSuccess) e = mark(2, dev->side);
     if (e == cudaSuccess && cascade)
-      e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, dev->side);
+      e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_cascade, true, dev->side, pdl);
     if (e == cudaSuccess) e = mark(3, dev->side);
+    if (e == cudaSuccess) e = launch_merge(p, merge_grid(), dev->side, pdl);
     if (e == cudaSuccess) e = cudaEventRecord(dev->ev_join, dev->side);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(s, dev->ev_join, 0);
-  }
-  if (e == cudaSuccess) {
-    const int want = (p.num_seqs * p.num_q_heads + 7) / 8;
-    const int grid = want < dev->sms * 8 ? (want > 0 ? want : 1) : dev->sms * 8;
-    e = launch_merge(p, grid, s);
   }
   if (e == cudaSuccess) e = mark(5, s);
   return from_cuda(e);
@@ -456,20 +465,23 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
     return ev ? cudaEventRecordWithFlags(reinterpret_cast<cudaEvent_t>(ev[i]), s, rec_flags) : cudaSuccess;
   };
   const bool cascade = p.cascade_enabled && p.window == 0;
-  // every kernel on `stream`: there is no append kernel to run beside
+  // every kernel on `stream`: there is no append kernel to run beside; the
+  // planner, the cascade pass and the merge are programmatic launches
+  // unless phase events are recorded between the kernels
+  const bool pdl = ev == nullptr;
   cudaError_t e = mark(0);
-  if (e == cudaSuccess) e = launch_plan(p, s);
+  if (e == cudaSuccess) e = launch_plan(p, s, pdl);
   if (e == cudaSuccess) e = mark(1);
-  if (e == cudaSuccess) e = launch_decode_fp8(kv8, p, dev->sms * dev->bpsm_fp8, false, s);
+  if (e == cudaSuccess) e = launch_decode_fp8(kv8, p, dev->sms * dev->bpsm_fp8, false, s, false);
   if (e == cudaSuccess) e = mark(2);
   if (e == cudaSuccess && cascade)
-    e = launch_decode_fp8(kv8, p, dev->sms * dev->bpsm_fp8_cascade, true, s);
+    e = launch_decode_fp8(kv8, p, dev->sms * dev->bpsm_fp8_cascade, true, s, pdl);
   if (e == cudaSuccess) e = mark(3);
   if (e == cudaSuccess) e = mark(4);
   if (e == cudaSuccess) {
     const int want = (p.num_seqs * p.num_q_heads + 7) / 8;
     const int grid = want < dev->sms * 8 ? (want > 0 ? want : 1) : dev->sms * 8;
-    e = launch_merge(p, grid, s);
+    e = launch_merge(p, grid, s, pdl);
   }
   if (e == cudaSuccess) e = mark(5);
   return from_cuda(e);
@@ -532,7 +544,7 @@ mcpu_status mcpu_selftest_append_abort(const void* q, const void* k_cache, const
   p.selftest_report = report;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(report, 0, 16 * sizeof(int64_t), s);
-  if (e == cudaSuccess) e = launch_plan(p, s);
+  if (e == cudaSuccess) e = launch_plan(p, s, false);
   if (e == cudaSuccess) e = launch_append_tc_selftest(kmap, vmap, qmap, p, s);
   return from_cuda(e);
 }

@@ -24,10 +24,10 @@
 #include "common.cuh"
 
 namespace mcpu {
-cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream);
+cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream, bool programmatic);
 cudaError_t prepare_plan_kernel();
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
-                          bool cascade, cudaStream_t stream);
+                          bool cascade, cudaStream_t stream, bool programmatic);
 cudaError_t prepare_decode_kernels(int* bpsm_decode, int* bpsm_cascade);
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                              const AttnParams& p, int grid, cudaStream_t stream);
@@ -177,8 +177,8 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
   // start at zero (the planner rewrites every other field it reads).
   // Every row writes its own output, so the log-sum-exp merge is not needed.
   cudaError_t e = cudaMemsetAsync(dev->scratch, 0, sizeof(int32_t), s);
-  if (e == cudaSuccess) e = launch_plan(p, s);
-  if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s);
+  if (e == cudaSuccess) e = launch_plan(p, s, false);
+  if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s, false);
   if (e == cudaSuccess) e = launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
   if (e == cudaSuccess && status_word)
     e = cudaMemcpyAsync(status_word, dev->scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s);

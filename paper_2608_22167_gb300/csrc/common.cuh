@@ -173,6 +173,15 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   return t;
 }
 
+// Programmatic dependent launch. A grid launched with programmatic stream
+// serialization may begin while the grid before it on the stream still
+// runs: grid_dep_wait() returns once that grid has completed and its memory
+// operations are visible (at once when the launch was an ordinary one), and
+// grid_dep_launch() lets the next grid of the stream launch before this one
+// has ended (a CTA that exits counts as having called it).
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
@@ -354,5 +363,27 @@ __device__ __forceinline__ float ex2_approx(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+
+// Launch configuration of one kernel, with programmatic stream serialization
+// when `programmatic` is set (the kernel then waits with grid_dep_wait()
+// before it uses the previous grid's results). Used in place: `cfg.attrs`
+// points into the object.
+struct LaunchCfg {
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  LaunchCfg(dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool programmatic) {
+    cfg = cudaLaunchConfig_t{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 1 : 0;
+  }
+  LaunchCfg(const LaunchCfg&) = delete;
+  LaunchCfg& operator=(const LaunchCfg&) = delete;
+};
 
 }  // namespace mcpu

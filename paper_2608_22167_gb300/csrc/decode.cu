@@ -36,7 +36,14 @@ template <int NT>
 __global__ void __launch_bounds__(kDecodeWarps * 32)
     decode_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                   const AttnParams p) {
-  if ((NT == 1 ? header(p)->n_decode : header(p)->n_cascade) == 0) return;  // nothing of this kind
+  // The cascade pass (NT > 1) may be launched programmatically after the
+  // decode kernel and run beside its tail: it reads nothing the decode
+  // kernel writes, but it waits for that kernel before it exits, so that its
+  // end still implies the decode kernel's (the merge comes after both).
+  if ((NT == 1 ? header(p)->n_decode : header(p)->n_cascade) == 0) {  // nothing of this kind
+    if (NT > 1) grid_dep_wait();
+    return;
+  }
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t raw = smem_addr(smem_raw);
@@ -293,6 +300,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     }
     if (timed_out) {
       raise_status(p, kStatusTimeout);
+      if (NT > 1) grid_dep_wait();
       return;  // the ring's phase tracking is lost: this warp stops here
     }
     seq += n;
@@ -355,15 +363,18 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     fence_proxy_async();
     __syncwarp();
   }
+  // no item left for this warp: the grid after this one may launch
+  grid_dep_launch();
+  if (NT > 1) grid_dep_wait();
 }
 
+// `programmatic` (cascade pass only): launched with programmatic stream
+// serialization right after the decode kernel on the same stream.
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttnParams& p, int grid,
-                          bool cascade, cudaStream_t stream) {
-  if (cascade)
-    decode_kernel<4><<<grid, kDecodeWarps * 32, decode_smem_bytes(), stream>>>(kmap, vmap, p);
-  else
-    decode_kernel<1><<<grid, kDecodeWarps * 32, decode_smem_bytes(), stream>>>(kmap, vmap, p);
-  return cudaGetLastError();
+                          bool cascade, cudaStream_t stream, bool programmatic) {
+  LaunchCfg lc(dim3(grid), dim3(kDecodeWarps * 32), decode_smem_bytes(), stream, programmatic && cascade);
+  return cascade ? cudaLaunchKernelEx(&lc.cfg, decode_kernel<4>, kmap, vmap, p)
+                 : cudaLaunchKernelEx(&lc.cfg, decode_kernel<1>, kmap, vmap, p);
 }
 
 cudaError_t prepare_decode_kernels(int* blocks_per_sm_decode, int* blocks_per_sm_cascade) {

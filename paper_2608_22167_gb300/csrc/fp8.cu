@@ -97,7 +97,12 @@ __device__ __forceinline__ uint32_t key_byte_mask(int c, int lo, int hi) {
 template <int NT>
 __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1)
     decode_fp8_kernel(const uint8_t* __restrict__ kv8, const AttnParams p) {
-  if ((NT == 1 ? header(p)->n_decode : header(p)->n_cascade) == 0) return;  // nothing of this kind
+  // The cascade pass (NT > 1) may be launched programmatically after the
+  // decode kernel: it waits for that kernel before it exits (see decode.cu).
+  if ((NT == 1 ? header(p)->n_decode : header(p)->n_cascade) == 0) {  // nothing of this kind
+    if (NT > 1) grid_dep_wait();
+    return;
+  }
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
@@ -403,6 +408,7 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1)
     }
     if (timed_out) {
       raise_status(p, kStatusTimeout);
+      if (NT > 1) grid_dep_wait();
       return;  // the ring's phase tracking is lost: this warp stops here
     }
     seq += n;
@@ -467,6 +473,9 @@ __global__ void __launch_bounds__(kF8Warps * 32, NT == 1 ? 4 : 1)
     fence_proxy_async();
     __syncwarp();
   }
+  // no item left for this warp: the grid after this one may launch
+  grid_dep_launch();
+  if (NT > 1) grid_dep_wait();
 }
 
 // ------------------------------------------------------------ fp8 KV append
@@ -575,13 +584,14 @@ cudaError_t launch_kv_append_fp8(const void* k_new, const void* v_new, void* kv8
   return cudaGetLastError();
 }
 
-cudaError_t launch_decode_fp8(const void* kv8, const AttnParams& p, int grid, bool cascade, cudaStream_t stream) {
+// `programmatic` (cascade pass only): launched with programmatic stream
+// serialization right after the decode kernel on the same stream.
+cudaError_t launch_decode_fp8(const void* kv8, const AttnParams& p, int grid, bool cascade, cudaStream_t stream,
+                              bool programmatic) {
   const uint8_t* pool = static_cast<const uint8_t*>(kv8);
-  if (cascade)
-    decode_fp8_kernel<4><<<grid, kF8Warps * 32, decode_fp8_smem_bytes(), stream>>>(pool, p);
-  else
-    decode_fp8_kernel<1><<<grid, kF8Warps * 32, decode_fp8_smem_bytes(), stream>>>(pool, p);
-  return cudaGetLastError();
+  LaunchCfg lc(dim3(grid), dim3(kF8Warps * 32), decode_fp8_smem_bytes(), stream, programmatic && cascade);
+  return cascade ? cudaLaunchKernelEx(&lc.cfg, decode_fp8_kernel<4>, pool, p)
+                 : cudaLaunchKernelEx(&lc.cfg, decode_fp8_kernel<1>, pool, p);
 }
 
 cudaError_t prepare_fp8_kernels(int* blocks_per_sm_decode, int* blocks_per_sm_cascade) {

@@ -23,6 +23,10 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParams p) {
+  // launched programmatically after the last kernel that writes partials:
+  // nothing is read before that kernel (and, through its own wait, every
+  // earlier one) has completed
+  grid_dep_wait();
   const PlanHeader* hdr = header(p);
   const int lane = threadIdx.x & 31;
   const int Hq = p.num_q_heads;
@@ -85,9 +89,9 @@ cudaError_t prepare_merge_kernel() {
                               cudaSharedmemCarveoutMaxShared);
 }
 
-cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream) {
-  merge_kernel<<<grid, kMergeWarps * 32, 0, stream>>>(p);
-  return cudaGetLastError();
+cudaError_t launch_merge(const AttnParams& p, int grid, cudaStream_t stream, bool programmatic) {
+  LaunchCfg lc(dim3(grid), dim3(kMergeWarps * 32), 0, stream, programmatic);
+  return cudaLaunchKernelEx(&lc.cfg, merge_kernel, p);
 }
 
 }  // namespace mcpu

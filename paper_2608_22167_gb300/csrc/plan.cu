@@ -147,6 +147,7 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
   }
   __syncthreads();
   if (sm.bad_global) {
+    grid_dep_wait();  // nothing of this call ends before the prefix scan
     if (tid == 0) {
       hdr->n_decode = hdr->n_cascade = hdr->n_append = hdr->n_merge = 0;
       hdr->n_parts = 0;
@@ -178,7 +179,10 @@ __global__ void __launch_bounds__(NT, 1) plan_kernel(AttnParams p) {
 
   // ---- phase 2: shared-prefix groups (full-context calls only)
   // lcp[r] = leading physical pages row r shares with row r - 1 (full pages
-  // of both), scanned beforehand by lcp_kernel across the whole GPU.
+  // of both), scanned beforehand by lcp_kernel across the whole GPU. The
+  // planner may have been launched while that scan ran (phase 1 reads only
+  // the caller's arrays): wait for it here.
+  grid_dep_wait();
   const bool cascade = p.cascade_enabled && p.window <= 0;
   if (cascade) {
     const int* lcp_ws = reinterpret_cast<const int*>(p.ws + p.lay.lcp);
@@ -470,6 +474,7 @@ constexpr int kLcpWarps = 8;
 constexpr int kLcpPerLane = 16;
 
 __global__ void __launch_bounds__(kLcpWarps * 32) lcp_kernel(const AttnParams p) {
+  grid_dep_launch();  // the planner may start its first phase meanwhile
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * kLcpWarps + (threadIdx.x >> 5);
   int* lcp = reinterpret_cast<int*>(p.ws + p.lay.lcp);
@@ -510,20 +515,22 @@ __global__ void __launch_bounds__(kLcpWarps * 32) lcp_kernel(const AttnParams p)
   if (lane == 0) lcp[r] = min(n, lim);
 }
 
-cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream) {
+cudaError_t launch_plan(const AttnParams& p, cudaStream_t stream, bool programmatic) {
   static_assert(sizeof(PlanSmem) < 200 * 1024, "planner shared memory");
-  if (p.cascade_enabled && p.window <= 0 && p.num_seqs > 0) {
+  const bool scan = p.cascade_enabled && p.window <= 0 && p.num_seqs > 0;
+  if (scan) {
     lcp_kernel<<<(p.num_seqs + kLcpWarps - 1) / kLcpWarps, kLcpWarps * 32, 0, stream>>>(p);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  // fewer threads for small batches: every phase ends in a CTA barrier, and
-  // barriers over 8 warps are cheaper than over 32
-  if (p.num_seqs <= R * 256)
-    plan_kernel<256><<<1, 256, sizeof(PlanSmem), stream>>>(p);
-  else
-    plan_kernel<kPlanThreads><<<1, kPlanThreads, sizeof(PlanSmem), stream>>>(p);
-  return cudaGetLastError();
+  // After the prefix scan (and only then: an earlier grid of the caller's
+  // may write what phase 1 reads) the planner may be launched
+  // programmatically, so that its launch and first phase overlap the scan.
+  // Fewer threads for small batches: every phase ends in a CTA barrier, and
+  // barriers over 8 warps are cheaper than over 32.
+  const bool small = p.num_seqs <= R * 256;
+  LaunchCfg lc(dim3(1), dim3(small ? 256 : kPlanThreads), sizeof(PlanSmem), stream, programmatic && scan);
+  return small ? cudaLaunchKernelEx(&lc.cfg, plan_kernel<256>, p) : cudaLaunchKernelEx(&lc.cfg, plan_kernel<kPlanThreads>, p);
 }
 
 cudaError_t prepare_plan_kernel() {
