@@ -21,7 +21,7 @@ cudaError_t launch_append(const CUtensorMap& kmap, const CUtensorMap& vmap, cons
                           cudaStream_t stream);
 cudaError_t prepare_append_kernel(int* bpsm);
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
-                             const AttnParams& p, int grid, cudaStream_t stream);
+                             const AttnParams& p, int grid, bool out_host, cudaStream_t stream);
 cudaError_t launch_append_tc_selftest(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                                       const AttnParams& p, cudaStream_t stream);
 cudaError_t prepare_append_tc_kernel(int* bpsm);
@@ -328,6 +328,9 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
     return ev ? cudaEventRecordWithFlags(reinterpret_cast<cudaEvent_t>(ev[i]), on, rec_flags) : cudaSuccess;
   };
   const bool serial = opts && (opts->flags & MCPU_FLAG_SERIAL);
+  // out and lse in page-locked host memory: the append kernel's form that
+  // writes whole rows over the host link
+  const bool out_host = opts && (opts->flags & MCPU_FLAG_HOST_OUT_DIRECT);
   const bool cascade = p.cascade_enabled && p.window == 0;
   // Programmatic launches (the planner after the prefix scan, the cascade
   // pass after the decode kernel, the merge after the cascade pass) overlap
@@ -340,7 +343,7 @@ mcpu_status mcpu_paged_attention_forward(const void* q, const void* k_cache, con
   };
   auto launch_append_kernel = [&]() -> cudaError_t {
     if (legacy_append) return launch_append(kmap, vmap, p, dev->sms * dev->bpsm_append, s);
-    return launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
+    return launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, out_host, s);
   };
   cudaError_t e = mark(0, s);
   if (e == cudaSuccess) e = launch_plan(p, s, pdl);

@@ -206,7 +206,17 @@ struct Slice {
   const void *q, *k_new, *v_new;
   void* out;
   float* lse;
+  bool out_host;  // out and lse are the caller's page-locked host buffers
 };
+
+// The caller's options for a slice's forward, with MCPU_FLAG_HOST_OUT_DIRECT
+// set exactly when that forward writes into host memory.
+mcpu_options slice_options(const mcpu_options* opts, const Slice& c) {
+  mcpu_options o = {};
+  if (opts) o = *opts;
+  o.flags = c.out_host ? (o.flags | MCPU_FLAG_HOST_OUT_DIRECT) : (o.flags & ~MCPU_FLAG_HOST_OUT_DIRECT);
+  return o;
+}
 
 // The pipeline shared by the bf16 and fp8 calls: checks, slicing, the
 // copies in and out on the stage's streams, and `compute(slice)` (the KV
@@ -309,6 +319,7 @@ mcpu_status host_call(mcpu_host_stage* hs, const void* q_host, const void* k_new
     c.v_new = sl.vn + t0 * kv_row;
     c.out = (out_direct ? out_direct : sl.out) + t0 * q_row;
     c.lse = reinterpret_cast<float*>((lse_direct ? lse_direct : reinterpret_cast<uint8_t*>(sl.lse)) + t0 * lse_row);
+    c.out_host = out_direct != nullptr;
     const mcpu_status st = compute(c);
     if (st != MCPU_OK) return fail_after_enqueue(hs, sl, s, st);
     if (out_direct) continue;  // written in place by the kernels
@@ -353,9 +364,10 @@ mcpu_status mcpu_paged_attention_host(mcpu_host_stage* hs, const void* q_host, c
                      mcpu_status st = mcpu_kv_append(c.k_new, c.v_new, k_cache, v_cache, c.block_table, c.seq_lens,
                                                      c.query_start_loc, &c.dims, status, stream);
                      if (st != MCPU_OK) return st;
+                     const mcpu_options o = slice_options(opts, c);
                      return mcpu_paged_attention_forward(c.q, k_cache, v_cache, c.block_table, c.seq_lens,
                                                          c.query_start_loc, sliding_window, softmax_scale, &c.dims,
-                                                         c.out, c.lse, workspace, workspace_bytes, opts, stream);
+                                                         c.out, c.lse, workspace, workspace_bytes, &o, stream);
                    });
 }
 
@@ -374,9 +386,10 @@ mcpu_status mcpu_paged_attention_host_fp8(mcpu_host_stage* hs, const void* q_hos
                      mcpu_status st = mcpu_kv_append_fp8(c.k_new, c.v_new, kv8, c.block_table, c.seq_lens,
                                                          c.query_start_loc, &c.dims, status, stream);
                      if (st != MCPU_OK) return st;
+                     const mcpu_options o = slice_options(opts, c);
                      return mcpu_paged_attention_forward_fp8(c.q, kv8, c.block_table, c.seq_lens, c.query_start_loc,
                                                              sliding_window, softmax_scale, &c.dims, c.out, c.lse,
-                                                             workspace, workspace_bytes, opts, stream);
+                                                             workspace, workspace_bytes, &o, stream);
                    });
 }
 

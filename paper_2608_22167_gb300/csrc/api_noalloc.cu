@@ -30,7 +30,7 @@ cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, cons
                           bool cascade, cudaStream_t stream, bool programmatic);
 cudaError_t prepare_decode_kernels(int* bpsm_decode, int* bpsm_cascade);
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
-                             const AttnParams& p, int grid, cudaStream_t stream);
+                             const AttnParams& p, int grid, bool out_host, cudaStream_t stream);
 cudaError_t prepare_append_tc_kernel(int* bpsm);
 }  // namespace mcpu
 
@@ -179,7 +179,7 @@ extern "C" mcpu_status mcpu_paged_attention_forward_noalloc(
   cudaError_t e = cudaMemsetAsync(dev->scratch, 0, sizeof(int32_t), s);
   if (e == cudaSuccess) e = launch_plan(p, s, false);
   if (e == cudaSuccess) e = launch_decode(kmap, vmap, p, dev->sms * dev->bpsm_decode, false, s, false);
-  if (e == cudaSuccess) e = launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, s);
+  if (e == cudaSuccess) e = launch_append_tc(kmap, vmap, qmap, p, dev->sms * dev->bpsm_append_tc, false, s);
   if (e == cudaSuccess && status_word)
     e = cudaMemcpyAsync(status_word, dev->scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, s);
   return from_cuda(e);

@@ -14,7 +14,10 @@
 //              rescales O (lazily: only when the max grows by more than 2^8;
 //              a rise inside the second chunk rescales the first chunk's P in
 //              place). The S buffer is released as soon as both chunks are in
-//              registers. Epilogue: O / l and the log-sum-exp to global memory;
+//              registers. Epilogue: O / l and the log-sum-exp to global memory
+//              (out in host memory, append_tc_kernel<*, true>: each warp's rows
+//              staged through 1 KiB of shared memory so that every store
+//              instruction writes four whole 128-byte rows);
 //   warp 8     TMA producer: item queue, both query tiles (one 3-D box of
 //              (256 / g) tokens x g heads x 64 dims), and K and V blocks
 //              (8 pages = 128 keys, 16 KiB) in two rings of their own: a K
@@ -43,7 +46,7 @@
 // A wait that runs out sets an abort flag in shared memory that every other
 // role's waits poll, so the whole CTA leaves within microseconds; before TMEM
 // is freed the issuers wait for their MMAs and the producer for its copies
-// still in flight. append_tc_kernel<true> is the self-test form of the same
+// still in flight. append_tc_kernel<true, false> is the self-test form of the same
 // kernel (mcpu_selftest_append_abort): one chosen role stops at the second
 // key block of its first item and waits on a barrier nothing completes (for
 // half the wait limit), and each warp reports when it left.
@@ -60,6 +63,7 @@ constexpr int kTcKStages = 4, kTcVStages = 3;
 constexpr int kTcQBytes = kAppendTcRows * kRowBytes;  // both tiles: 32 KiB
 constexpr int kTcTileQBytes = kTcRows * kRowBytes;    // 16 KiB
 constexpr int kTcKvBytes = kTcKeys * kRowBytes;       // one K or V block: 16 KiB
+constexpr int kTcStageBytes = 8 * kRowBytes;          // out-in-host-memory form: output staging per softmax warp
 constexpr int kTcProducerWarp = 8, kTcSWarp = 9, kTcPvWarp = 10;
 constexpr int kTcThreads = 352;
 constexpr uint32_t kTmemCols = 512;
@@ -85,8 +89,9 @@ struct TcSmem {  // barriers and small state, after the tiles
   uint64_t t_start;    // self-test form only: %globaltimer at kernel start
 };
 
-size_t append_tc_smem_bytes() {
-  return 1024 + kTcQBytes + (size_t)(kTcKStages + kTcVStages) * kTcKvBytes + sizeof(TcSmem);
+size_t append_tc_smem_bytes(bool out_host) {
+  return 1024 + kTcQBytes + (size_t)(kTcKStages + kTcVStages) * kTcKvBytes + (out_host ? 8 * kTcStageBytes : 0) +
+         sizeof(TcSmem);
 }
 
 namespace {
@@ -170,6 +175,14 @@ __device__ __forceinline__ float chunk_exp(const uint32_t (&sv)[2][32], float sc
 __device__ __forceinline__ void st_shared_zero16(uint32_t addr) {
   asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(addr), "r"(0u) : "memory");
 }
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
+  return v;
+}
 
 // Self-test form only: the stalled role waits on a barrier nothing completes
 // for half the library's wait limit, without polling the abort flag; then it
@@ -214,7 +227,8 @@ __device__ __forceinline__ float chunk_probs(const uint32_t (&sv)[2][32], float 
 
 }  // namespace
 
-template <bool kSelfTest>
+// kOutHost: out lies in page-locked host memory (written over the host link)
+template <bool kSelfTest, bool kOutHost>
 __global__ void __maxnreg__(144)
     append_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap qmap, const AttnParams p) {
@@ -227,8 +241,9 @@ __global__ void __maxnreg__(144)
   const uint32_t sQ = base;
   const uint32_t sK = base + kTcQBytes;
   const uint32_t sV = sK + kTcKStages * kTcKvBytes;
+  const uint32_t sStage = sV + kTcVStages * kTcKvBytes;  // kOutHost only: 8 x 1 KiB, one per softmax warp
   TcSmem& st = *reinterpret_cast<TcSmem*>(smem_raw + (base - raw) + kTcQBytes +
-                                          (kTcKStages + kTcVStages) * kTcKvBytes);
+                                          (kTcKStages + kTcVStages) * kTcKvBytes + (kOutHost ? 8 * kTcStageBytes : 0));
   volatile int32_t* abort_flag = &st.abort_flag;
   auto bar = [&](uint64_t& b) { return smem_addr(&b); };
 
@@ -617,7 +632,48 @@ __global__ void __maxnreg__(144)
         mbar_arrive(bar(st.o_free[x]));
         mbar_arrive(bar(st.item_empty[slot]));
       }
-      if (valid) {
+      if constexpr (kOutHost) {
+        // O / l as bf16, this thread's row in 32 words (dims 2j, 2j + 1)
+        float inv = l > 0.f ? 1.f / l : 0.f;
+        float lse2 = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
+        if (p.sinks != nullptr) inv = finish_with_sink(m_ref, l, sink_log2(p, kvh * g + head), &lse2);
+        uint32_t w[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          w[j] = pack_bf16x2(__uint_as_float(ov[j >> 4][2 * (j & 15)]) * inv,
+                             __uint_as_float(ov[j >> 4][2 * (j & 15) + 1]) * inv);
+        // The rows cross the host link: they go out through this warp's
+        // 1 KiB of shared memory, 8 rows per round (16-byte chunk c of
+        // staged row r at r * 128 + (c ^ r) * 16, no bank conflicts on
+        // either side), so that each store instruction writes 4 whole
+        // 128-byte rows instead of a 16-byte piece of 32 rows.
+        const uint32_t stg = sStage + warp * kTcStageBytes;
+        const int rr = lane >> 3, c = lane & 7;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if (rr == k) {
+            const int r = lane & 7;
+#pragma unroll
+            for (int cc = 0; cc < 8; ++cc)
+              st_shared_v4(stg + r * kRowBytes + ((cc ^ r) << 4), w[4 * cc], w[4 * cc + 1], w[4 * cc + 2],
+                           w[4 * cc + 3]);
+          }
+          __syncwarp();
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int r = rr + 4 * h;               // staged row
+            const int wrow = wq * 32 + 8 * k + r;   // its tile row
+            const int t = x * tile_tok + wrow / g;  // its token in the item
+            const uint4 v = ld_shared_v4(stg + r * kRowBytes + ((c ^ r) << 4));
+            if (t < a.n_tok) {
+              const size_t orow = (size_t)(a.token_begin + t) * Hq + kvh * g + wrow % g;
+              reinterpret_cast<uint4*>(p.out + orow * kHeadDim)[c] = v;
+            }
+          }
+          __syncwarp();  // the next round overwrites the staging rows
+        }
+        if (valid) p.lse[(size_t)(a.token_begin + tok) * Hq + kvh * g + head] = lse2 * 0.69314718055994531f;
+      } else if (valid) {
         float inv = l > 0.f ? 1.f / l : 0.f;
         float lse2 = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
         if (p.sinks != nullptr) inv = finish_with_sink(m_ref, l, sink_log2(p, kvh * g + head), &lse2);
@@ -656,9 +712,13 @@ __global__ void __maxnreg__(144)
   }
 }
 
+// out_host: p.out is page-locked host memory (the staged-store form).
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
-                             const AttnParams& p, int grid, cudaStream_t stream) {
-  append_tc_kernel<false><<<grid, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
+                             const AttnParams& p, int grid, bool out_host, cudaStream_t stream) {
+  if (out_host)
+    append_tc_kernel<false, true><<<grid, kTcThreads, append_tc_smem_bytes(true), stream>>>(kmap, vmap, qmap, p);
+  else
+    append_tc_kernel<false, false><<<grid, kTcThreads, append_tc_smem_bytes(false), stream>>>(kmap, vmap, qmap, p);
   return cudaGetLastError();
 }
 
@@ -666,19 +726,19 @@ cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, c
 // p.selftest_report receives the abort flag and each warp's exit time.
 cudaError_t launch_append_tc_selftest(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                                       const AttnParams& p, cudaStream_t stream) {
-  append_tc_kernel<true><<<1, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
+  append_tc_kernel<true, false><<<1, kTcThreads, append_tc_smem_bytes(false), stream>>>(kmap, vmap, qmap, p);
   return cudaGetLastError();
 }
 
 cudaError_t prepare_append_tc_kernel(int* blocks_per_sm) {
-  for (auto fn : {append_tc_kernel<false>, append_tc_kernel<true>}) {
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_tc_smem_bytes());
+  for (auto fn : {append_tc_kernel<false, false>, append_tc_kernel<true, false>, append_tc_kernel<false, true>}) {
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_tc_smem_bytes(true));
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
   }
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_tc_kernel<false>, kTcThreads,
-                                                       append_tc_smem_bytes());
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_tc_kernel<false, false>, kTcThreads,
+                                                       append_tc_smem_bytes(false));
 }
 
 }  // namespace mcpu
