@@ -581,13 +581,14 @@ def run_ours(args, rank, world, dev):
         torch.cuda.synchronize()
         other_ms = o0.elapsed_time(o1) / n_other
 
-    # per-kernel times, ms per step. Decode then cascade run on the library's
-    # side stream concurrently with the append kernel: events [1]->[2]
-    # decode, [2]->[3] cascade (side stream), [1]->[4] append; the merge
-    # starts at the join, the later of [3] and [4].
+    # per-kernel times, ms per step. Decode, cascade and merge run in that
+    # order on the library's side stream concurrently with the append
+    # kernel: events [1]->[2] decode, [2]->[3] cascade (side stream), [1]->[4]
+    # append, [5] after the join; "merge" is the time from the later of [3]
+    # and [4] to [5], what the merge (and the join) add past both.
     ktime = {n: 0.0 for n in ("plan", "decode", "cascade", "append_chunk", "merge")}
     layer_ms = [0.0] * nl  # each layer's forward span (planner to merge)
-    layer_k = [[0.0] * 5 for _ in range(nl)]  # plan, decode+cascade, append, merge (from the join), total
+    layer_k = [[0.0] * 5 for _ in range(nl)]  # plan, decode+cascade, append, merge (past both), total
     for k in range(n_sets):
         for i in range(nl):
             ev = phase[k][i]

@@ -1,8 +1,9 @@
 // C ABI of the paged-attention path (declared in include/mcpu.h): host-side
 // argument checks, per-device one-time setup (kernel attributes, occupancy),
 // TMA descriptors of the two KV pools, and the launch sequence
-//   planner -> cascade pass -> split-KV decode -> append-chunk -> LSE merge
-// on the caller's stream. Nothing here allocates device memory.
+//   prefix scan -> planner -> append-chunk kernel, and beside it on a side
+//   stream: split-KV decode -> cascade pass -> LSE merge
+// forked from and joined back into the caller's stream. Nothing here allocates device memory.
 #include <cudaTypedefs.h>
 
 #include <mutex>
