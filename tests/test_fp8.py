@@ -370,3 +370,33 @@ def test_cuda_graph_replay():
                                         h["softmax_scale"])
     go, gl = run.out_host()
     assert_parity(go, gl, oracle.bf16_bits_to_float(ro), rl, "fp8 graph replay")
+
+
+def test_programmatic_launches_match_ordinary_ones_bitwise():
+    # fp8 chain on one stream: the planner, the cascade pass (after the
+    # decode kernel) and the merge (after the cascade pass) are programmatic
+    # launches unless phase events are recorded; both forms, and a graph of
+    # the programmatic one, agree bit for bit on groups with split rows
+    b = _grouped(7)
+    run, _ = _full_check(b, split_pages=2, what="fp8 programmatic")
+    assert run.header()["n_cascade"] > 0 and run.header()["n_merge"] > 0
+    out_p, lse_p = run.out_host()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(mcpu.NUM_PHASE_EVENTS)]
+    for e in ev:  # torch creates the CUDA event at its first record
+        e.record()
+    run.out.fill_(float("nan"))
+    mcpu.mcpu_paged_attention_forward_fp8(run.q, run.kv8, run.bt, run.sl, run.qsl, run.window, b.softmax_scale,
+                                          run.out, run.lse, run.ws, split_pages=2, phase_events=ev)
+    torch.cuda.synchronize()
+    assert run.status()[0] == 0
+    out_o, lse_o = run.out_host()
+    assert np.array_equal(out_p, out_o) and np.array_equal(lse_p, lse_o)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        run.forward(split_pages=2)
+    run.out.fill_(float("nan"))
+    g.replay()
+    torch.cuda.synchronize()
+    assert run.status()[0] == 0
+    out_g, lse_g = run.out_host()
+    assert np.array_equal(out_p, out_g) and np.array_equal(lse_p, lse_g)

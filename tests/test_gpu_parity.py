@@ -533,3 +533,41 @@ def test_largest_row_count():
     assert run.status()[0] == 0
     rows = sorted(rng.choice(B, size=40, replace=False))
     _good_rows_parity(run, b, rows, "2048 rows")
+
+
+@pytest.mark.parametrize("layer", [0, 1])
+def test_programmatic_launches_match_ordinary_ones_bitwise(layer):
+    # Without phase events the planner (after the prefix scan), the cascade
+    # pass (after the decode kernel) and the merge (after the cascade pass)
+    # are programmatic launches that overlap the grid before them; with phase
+    # events every kernel is an ordinary launch. Layer 1 of the rollout
+    # profiling batch has GRPO groups (cascade items) and split rows; layer 0
+    # is a sliding-window layer. Results must agree bit for bit, eagerly and
+    # as a replayed CUDA graph of the programmatic form.
+    b = W.config_rollout_small(device="cpu")
+    run = Run(b, layer)
+    run.append()
+    run.forward()
+    assert run.status()[0] == 0
+    if layer == 1:
+        assert run.header()["n_cascade"] > 0 and run.header()["n_merge"] > 0
+    out_p, lse_p = run.out_host()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(mcpu.NUM_PHASE_EVENTS)]
+    for e in ev:  # torch creates the CUDA event at its first record
+        e.record()
+    run.out.fill_(float("nan"))
+    mcpu.mcpu_paged_attention_forward(run.q, run.kc, run.vc, run.bt, run.sl, run.qsl, run.window,
+                                      b.softmax_scale, run.out, run.lse, run.ws, phase_events=ev)
+    torch.cuda.synchronize()
+    assert run.status()[0] == 0
+    out_o, lse_o = run.out_host()
+    assert np.array_equal(out_p, out_o) and np.array_equal(lse_p, lse_o)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        run.forward()
+    run.out.fill_(float("nan"))
+    g.replay()
+    torch.cuda.synchronize()
+    assert run.status()[0] == 0
+    out_g, lse_g = run.out_host()
+    assert np.array_equal(out_p, out_g) and np.array_equal(lse_p, lse_g)
