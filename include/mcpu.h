@@ -102,7 +102,7 @@ typedef struct mcpu_dims {
 #define MCPU_FLAG_MMA_SYNC_APPEND 0x2u  /* append chunks on the mma.sync kernel instead of tcgen05 */
 #define MCPU_FLAG_SERIAL 0x4u           /* run every kernel on `stream` (no side stream) */
 #define MCPU_FLAG_HOST_OUT_DIRECT 0x8u  /* host-buffer calls: kernels write out/lse straight into page-locked host memory;
-                                           forward calls: out/lse are page-locked host memory, written in whole rows */
+                                           forward calls: out/lse are page-locked host memory, written in whole sectors */
 typedef struct mcpu_options {
   uint32_t flags;             /* MCPU_FLAG_* */
   int32_t split_pages;        /* > 0: KV split length of decode rows, in pages (0 = auto) */
@@ -168,10 +168,10 @@ mcpu_status mcpu_kv_append(const void* k_new, const void* v_new, void* k_cache, 
  * planner and joins back at the end, with CUDA events. Pass
  * MCPU_FLAG_SERIAL to keep every kernel on `stream`. Set
  * MCPU_FLAG_HOST_OUT_DIRECT when out and lse are page-locked host memory
- * the device can address: the append kernel then writes out in whole
- * 128-byte rows, staged through 8 KiB more shared memory, which the host
- * link takes far better than 16-byte pieces of many rows (device memory
- * gives the same results that way, a little more slowly). The call is capturable in a CUDA graph (with mcpu_kv_append
+ * the device can address: the append kernel then writes out in 32-byte
+ * pieces (whole sectors, if out is 32-byte aligned), which the host link
+ * takes far better than 16-byte halves of sectors (device memory gives the
+ * same results that way). The call is capturable in a CUDA graph (with mcpu_kv_append
  * before it): it allocates nothing, synchronises nothing, and its work plan
  * is rebuilt on the device at every replay, so a replayed graph follows
  * changed seq_lens / block_table / query_start_loc contents as long as the

@@ -15,9 +15,8 @@
 //              a rise inside the second chunk rescales the first chunk's P in
 //              place). The S buffer is released as soon as both chunks are in
 //              registers. Epilogue: O / l and the log-sum-exp to global memory
-//              (out in host memory, append_tc_kernel<*, true>: each warp's rows
-//              staged through 1 KiB of shared memory so that every store
-//              instruction writes four whole 128-byte rows);
+//              (out in host memory, append_tc_kernel<*, true>: each row as
+//              four 32-byte stores, whole sectors for the host link);
 //   warp 8     TMA producer: item queue, both query tiles (one 3-D box of
 //              (256 / g) tokens x g heads x 64 dims), and K and V blocks
 //              (8 pages = 128 keys, 16 KiB) in two rings of their own: a K
@@ -63,7 +62,6 @@ constexpr int kTcKStages = 4, kTcVStages = 3;
 constexpr int kTcQBytes = kAppendTcRows * kRowBytes;  // both tiles: 32 KiB
 constexpr int kTcTileQBytes = kTcRows * kRowBytes;    // 16 KiB
 constexpr int kTcKvBytes = kTcKeys * kRowBytes;       // one K or V block: 16 KiB
-constexpr int kTcStageBytes = 8 * kRowBytes;          // out-in-host-memory form: output staging per softmax warp
 constexpr int kTcProducerWarp = 8, kTcSWarp = 9, kTcPvWarp = 10;
 constexpr int kTcThreads = 352;
 constexpr uint32_t kTmemCols = 512;
@@ -89,9 +87,8 @@ struct TcSmem {  // barriers and small state, after the tiles
   uint64_t t_start;    // self-test form only: %globaltimer at kernel start
 };
 
-size_t append_tc_smem_bytes(bool out_host) {
-  return 1024 + kTcQBytes + (size_t)(kTcKStages + kTcVStages) * kTcKvBytes + (out_host ? 8 * kTcStageBytes : 0) +
-         sizeof(TcSmem);
+size_t append_tc_smem_bytes() {
+  return 1024 + kTcQBytes + (size_t)(kTcKStages + kTcVStages) * kTcKvBytes + sizeof(TcSmem);
 }
 
 namespace {
@@ -175,13 +172,10 @@ __device__ __forceinline__ float chunk_exp(const uint32_t (&sv)[2][32], float sc
 __device__ __forceinline__ void st_shared_zero16(uint32_t addr) {
   asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(addr), "r"(0u) : "memory");
 }
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
-__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
-  uint4 v;
-  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
-  return v;
+// one 32-byte store (p 32-byte aligned)
+__device__ __forceinline__ void st_global_v8(void* p, const uint32_t* w) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+               "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7]) : "memory");
 }
 
 // Self-test form only: the stalled role waits on a barrier nothing completes
@@ -241,9 +235,8 @@ __global__ void __maxnreg__(144)
   const uint32_t sQ = base;
   const uint32_t sK = base + kTcQBytes;
   const uint32_t sV = sK + kTcKStages * kTcKvBytes;
-  const uint32_t sStage = sV + kTcVStages * kTcKvBytes;  // kOutHost only: 8 x 1 KiB, one per softmax warp
   TcSmem& st = *reinterpret_cast<TcSmem*>(smem_raw + (base - raw) + kTcQBytes +
-                                          (kTcKStages + kTcVStages) * kTcKvBytes + (kOutHost ? 8 * kTcStageBytes : 0));
+                                          (kTcKStages + kTcVStages) * kTcKvBytes);
   volatile int32_t* abort_flag = &st.abort_flag;
   auto bar = [&](uint64_t& b) { return smem_addr(&b); };
 
@@ -633,46 +626,30 @@ __global__ void __maxnreg__(144)
         mbar_arrive(bar(st.item_empty[slot]));
       }
       if constexpr (kOutHost) {
-        // O / l as bf16, this thread's row in 32 words (dims 2j, 2j + 1)
+        // O / l as bf16, this thread's row in 32 words (dims 2j, 2j + 1),
+        // written as four 32-byte pieces (whole sectors) when out is 32-byte
+        // aligned, else eight 16-byte ones
         float inv = l > 0.f ? 1.f / l : 0.f;
         float lse2 = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
         if (p.sinks != nullptr) inv = finish_with_sink(m_ref, l, sink_log2(p, kvh * g + head), &lse2);
-        uint32_t w[32];
+        if (valid) {
+          uint32_t w[32];
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-          w[j] = pack_bf16x2(__uint_as_float(ov[j >> 4][2 * (j & 15)]) * inv,
-                             __uint_as_float(ov[j >> 4][2 * (j & 15) + 1]) * inv);
-        // The rows cross the host link: they go out through this warp's
-        // 1 KiB of shared memory, 8 rows per round (16-byte chunk c of
-        // staged row r at r * 128 + (c ^ r) * 16, no bank conflicts on
-        // either side), so that each store instruction writes 4 whole
-        // 128-byte rows instead of a 16-byte piece of 32 rows.
-        const uint32_t stg = sStage + warp * kTcStageBytes;
-        const int rr = lane >> 3, c = lane & 7;
+          for (int j = 0; j < 32; ++j)
+            w[j] = pack_bf16x2(__uint_as_float(ov[j >> 4][2 * (j & 15)]) * inv,
+                               __uint_as_float(ov[j >> 4][2 * (j & 15) + 1]) * inv);
+          const size_t orow = (size_t)(a.token_begin + tok) * Hq + kvh * g + head;
+          uint8_t* dst = reinterpret_cast<uint8_t*>(p.out + orow * kHeadDim);
+          if ((reinterpret_cast<uintptr_t>(p.out) & 31) == 0) {
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          if (rr == k) {
-            const int r = lane & 7;
+            for (int q = 0; q < 4; ++q) st_global_v8(dst + 32 * q, w + 8 * q);
+          } else {
 #pragma unroll
-            for (int cc = 0; cc < 8; ++cc)
-              st_shared_v4(stg + r * kRowBytes + ((cc ^ r) << 4), w[4 * cc], w[4 * cc + 1], w[4 * cc + 2],
-                           w[4 * cc + 3]);
+            for (int q = 0; q < 8; ++q)
+              reinterpret_cast<uint4*>(dst)[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
           }
-          __syncwarp();
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int r = rr + 4 * h;               // staged row
-            const int wrow = wq * 32 + 8 * k + r;   // its tile row
-            const int t = x * tile_tok + wrow / g;  // its token in the item
-            const uint4 v = ld_shared_v4(stg + r * kRowBytes + ((c ^ r) << 4));
-            if (t < a.n_tok) {
-              const size_t orow = (size_t)(a.token_begin + t) * Hq + kvh * g + wrow % g;
-              reinterpret_cast<uint4*>(p.out + orow * kHeadDim)[c] = v;
-            }
-          }
-          __syncwarp();  // the next round overwrites the staging rows
+          p.lse[orow] = lse2 * 0.69314718055994531f;
         }
-        if (valid) p.lse[(size_t)(a.token_begin + tok) * Hq + kvh * g + head] = lse2 * 0.69314718055994531f;
       } else if (valid) {
         float inv = l > 0.f ? 1.f / l : 0.f;
         float lse2 = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
@@ -712,13 +689,13 @@ __global__ void __maxnreg__(144)
   }
 }
 
-// out_host: p.out is page-locked host memory (the staged-store form).
+// out_host: p.out is page-locked host memory (the form that writes whole sectors).
 cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                              const AttnParams& p, int grid, bool out_host, cudaStream_t stream) {
   if (out_host)
-    append_tc_kernel<false, true><<<grid, kTcThreads, append_tc_smem_bytes(true), stream>>>(kmap, vmap, qmap, p);
+    append_tc_kernel<false, true><<<grid, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
   else
-    append_tc_kernel<false, false><<<grid, kTcThreads, append_tc_smem_bytes(false), stream>>>(kmap, vmap, qmap, p);
+    append_tc_kernel<false, false><<<grid, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
   return cudaGetLastError();
 }
 
@@ -726,19 +703,19 @@ cudaError_t launch_append_tc(const CUtensorMap& kmap, const CUtensorMap& vmap, c
 // p.selftest_report receives the abort flag and each warp's exit time.
 cudaError_t launch_append_tc_selftest(const CUtensorMap& kmap, const CUtensorMap& vmap, const CUtensorMap& qmap,
                                       const AttnParams& p, cudaStream_t stream) {
-  append_tc_kernel<true, false><<<1, kTcThreads, append_tc_smem_bytes(false), stream>>>(kmap, vmap, qmap, p);
+  append_tc_kernel<true, false><<<1, kTcThreads, append_tc_smem_bytes(), stream>>>(kmap, vmap, qmap, p);
   return cudaGetLastError();
 }
 
 cudaError_t prepare_append_tc_kernel(int* blocks_per_sm) {
   for (auto fn : {append_tc_kernel<false, false>, append_tc_kernel<true, false>, append_tc_kernel<false, true>}) {
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_tc_smem_bytes(true));
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_tc_smem_bytes());
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
   }
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, append_tc_kernel<false, false>, kTcThreads,
-                                                       append_tc_smem_bytes(false));
+                                                       append_tc_smem_bytes());
 }
 
 }  // namespace mcpu

@@ -128,11 +128,10 @@ def test_direct_outputs_equal_the_staged_ones_bitwise(pinned):
 @pytest.mark.parametrize("hq,hkv", [(64, 8), (32, 8), (16, 8), (8, 8)])
 def test_forward_into_host_memory_equals_device_outputs_bitwise(hq, hkv, window):
     # MCPU_FLAG_HOST_OUT_DIRECT on a forward call: out and lse are page-locked
-    # host memory, and the append kernel writes whole rows staged through
-    # shared memory (each warp's 32 rows in 4 rounds of 8, every row mapped
-    # back to its token and head: g = 8, 4, 2, 1 and partial last tiles
-    # here). The values are those of the device-output form, bit for bit;
-    # rows past a tile's last token are never written.
+    # host memory, and the append kernel writes each row as four 32-byte
+    # stores (eight 16-byte ones when out is only 16-byte aligned, the second
+    # buffer here): g = 8, 4, 2, 1 and partial last tiles. The values are
+    # those of the device-output form, bit for bit.
     seq = np.array([900, 40, 2500, 16, 700, 333, 77])
     ql = np.array([1, 17, 300, 1, 45, 333, 5])
     b = W.build_batch("host_out", 3400 + hq + window, seq, ql, hq, hkv, layer_windows=(window,))
@@ -149,15 +148,20 @@ def test_forward_into_host_memory_equals_device_outputs_bitwise(hq, hkv, window)
     out_d = torch.full_like(q, float("nan"))
     lse_d = torch.full(q.shape[:2], float("nan"), dtype=torch.float32, device="cuda")
     mcpu.mcpu_paged_attention_forward(q, kc, vc, bt, sl, qsl, window, b.softmax_scale, out_d, lse_d, ws)
-    out_h = torch.full(q.shape, float("nan"), dtype=torch.bfloat16).pin_memory()
-    lse_h = torch.full(q.shape[:2], float("nan"), dtype=torch.float32).pin_memory()
-    mcpu.mcpu_paged_attention_forward(q, kc, vc, bt, sl, qsl, window, b.softmax_scale, out_h, lse_h, ws,
-                                      flags=mcpu.FLAG_HOST_OUT_DIRECT)
-    torch.cuda.synchronize()
-    code, bits = mcpu.mcpu_read_device_status(ws)
-    assert code == 0, bits
-    assert torch.equal(out_h.view(torch.int16), out_d.cpu().view(torch.int16))
-    assert torch.equal(lse_h, lse_d.cpu())
+    n = q.numel()
+    big = torch.full((n + 16,), float("nan"), dtype=torch.bfloat16).pin_memory()
+    assert big.data_ptr() % 32 == 0
+    for off in (0, 8):  # 32-byte aligned, then 16 bytes past it
+        out_h = big[off:off + n].view(q.shape)
+        out_h.fill_(float("nan"))
+        lse_h = torch.full(q.shape[:2], float("nan"), dtype=torch.float32).pin_memory()
+        mcpu.mcpu_paged_attention_forward(q, kc, vc, bt, sl, qsl, window, b.softmax_scale, out_h, lse_h, ws,
+                                          flags=mcpu.FLAG_HOST_OUT_DIRECT)
+        torch.cuda.synchronize()
+        code, bits = mcpu.mcpu_read_device_status(ws)
+        assert code == 0, bits
+        assert torch.equal(out_h.view(torch.int16), out_d.cpu().view(torch.int16)), off
+        assert torch.equal(lse_h, lse_d.cpu()), off
     if hq == 64:  # the device-output form is checked against the oracle elsewhere for every g
         ref_out, ref_lse = oracle_full(b, 0)[:2]
         assert_parity(out_h.float().numpy(), lse_h.numpy(), ref_out, ref_lse, f"host outputs W={window}")
