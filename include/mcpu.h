@@ -342,7 +342,9 @@ mcpu_status mcpu_paged_attention_forward_fp8(const void* q, const void* kv8, con
  * copied back (slices = 0 then means one slice). That suits the call whose
  * outputs are wanted right after it (nothing is left to copy once its last
  * kernel ends); a call followed by more work does better with the copies,
- * which run beside that work. Without the flag, or for other host memory,
+ * which run beside that work, and with slices = 1 (its output copy already
+ * overlaps the next call, and each slice adds its own planner and kernel
+ * tails). Without the flag, or for other host memory,
  * the outputs are staged and copied. Shared-prefix
  * detection only sees rows within one slice. query_start_loc_host is read
  * on the host during the call; the other host buffers are read or written
