@@ -1051,7 +1051,12 @@ def main():
         torch.cuda.set_device(dev)
         from __graft_entry__ import build
 
+        # one compile at most: rank 0 first, the others find it up to date
+        if world > 1 and rank != 0:
+            torch.distributed.barrier()
         build()
+        if world > 1 and rank == 0:
+            torch.distributed.barrier()
         res = run_churn(args, rank, world, dev) if args.workload == "churn" else run_ours(args, rank, world, dev)
         if (world == 1 and args.workload == "mixed" and args.kv == "bf16" and args.other_configs
                 and args.launch == "graph"):
