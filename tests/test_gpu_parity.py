@@ -571,3 +571,40 @@ def test_programmatic_launches_match_ordinary_ones_bitwise(layer):
     assert run.status()[0] == 0
     out_g, lse_g = run.out_host()
     assert np.array_equal(out_p, out_g) and np.array_equal(lse_p, lse_g)
+
+
+def _random_batch(seed):
+    """Decode and append rows of random lengths, sometimes GRPO groups sharing
+    prompt pages, sometimes a window; GQA group 8, 4, 2 or 1."""
+    rng = np.random.default_rng(seed)
+    groups, gs, B0 = int(rng.integers(0, 4)), int(rng.choice([2, 4, 8])), int(rng.integers(4, 24))
+    S = rng.integers(1, 6000, size=B0)
+    L = np.where(rng.random(B0) < 0.6, 1, np.minimum(S, rng.integers(2, 400, size=B0)))
+    kw = {}
+    if groups:
+        prompt = np.repeat(rng.integers(40, 2500, size=groups), gs)
+        Sg = prompt + rng.integers(1, 1500, size=groups * gs)
+        Lg = np.minimum(np.where(rng.random(groups * gs) < 0.8, 1, rng.integers(2, 100, size=groups * gs)), Sg)
+        S, L = np.concatenate([Sg, S]), np.concatenate([Lg, L])
+        kw = dict(shared_prefix_pages=np.concatenate([prompt // 16, np.zeros(B0, np.int64)]),
+                  prompt_lens=np.concatenate([prompt, np.zeros(B0, np.int64)]),
+                  group_of_row=np.concatenate([np.repeat(np.arange(groups), gs), -np.ones(B0, np.int64)]))
+    hq, hkv = [(64, 8), (32, 8), (16, 8), (8, 8)][int(rng.integers(0, 4))]
+    win = int(rng.choice([0, 0, 0, 128, 1000])) if not groups else 0
+    sinks = rng.normal(0, 2, size=hq).astype(np.float32) if seed % 3 == 0 else None
+    return W.build_batch("random", seed, S, L, hq, hkv, layer_windows=(win,), **kw), sinks
+
+
+@pytest.mark.parametrize("seed", [9001, 9003, 9005, 9007, 9008, 9014])
+def test_random_batches_with_groups_windows_and_sinks(seed):
+    # seeds chosen for: window 128 (g 2), groups + sinks (g 8), groups (g 8),
+    # groups (g 4), window 1000 (g 8), plain (g 1); each against the oracle on
+    # all outputs, the pools bit for bit, and the side-stream and
+    # single-stream launch orders bit for bit against each other
+    b, sinks = _random_batch(seed)
+    run, _ = _full_check(b, sinks=sinks, what=f"random{seed}")
+    out1, lse1 = run.out_host()
+    run.forward(flags=mcpu.FLAG_SERIAL, sinks=sinks)
+    assert run.status()[0] == 0
+    out2, lse2 = run.out_host()
+    assert np.array_equal(out1, out2) and np.array_equal(lse1, lse2)
